@@ -1,0 +1,79 @@
+"""Planted mistakes: each mutation below is a plausible error in the oracle (a dropped term, a
+wrong sign or index, a transposed operand, another rounding). It is applied to a temporary copy
+of ``oracle/voxzip_oracle.c``, compiled, and the pins must reject that copy. CPU only; the
+committed oracle is never modified."""
+import os
+
+import pytest
+
+import oracle
+import oracle_pins
+
+MUTATIONS = [
+    ("decay dropped", "score[j] *= gamma;", "score[j] *= 1.0;"),
+    ("decay applied twice", "score[j] *= gamma;", "score[j] *= gamma * gamma;"),
+    ("logit scale squared", "logit[j] = dot * scale;", "logit[j] = dot * scale * scale;"),
+    ("softmax denominator off", "const double p = exp(logit[j] - m) / z;",
+     "const double p = exp(logit[j] - m) / (z + 1.0);"),
+    ("new token score not zero-padded", "score[n] = 0.0;", "score[n] = 1.0;"),
+    ("append position off by one", "pos[n] = new_pos;", "pos[n] = new_pos + 1;"),
+    ("PV reads K instead of V", "oh[d] += p * V[(int64_t)j * D + d];",
+     "oh[d] += p * K[(int64_t)j * D + d];"),
+    ("query reversed against key", "dot += qh[d] * K[(int64_t)j * D + d];",
+     "dot += qh[D - 1 - d] * K[(int64_t)j * D + d];"),
+    ("ceil group boundaries (short groups last)",
+     "const int64_t lo = s + (j * l) / g;\n                const int64_t hi = s + ((j + 1) * l) / g;",
+     "const int64_t lo = s + (j * l + g - 1) / g;\n                const int64_t hi = s + ((j + 1) * l + g - 1) / g;"),
+    ("group count not clamped to span length", "span_groups[i] < l ? span_groups[i] : l",
+     "span_groups[i]"),
+    ("anchor row ignores the group index", "anchor[(anchor_row + j) * D + d]",
+     "anchor[(anchor_row) * D + d]"),
+    ("empty spans' anchor rows not counted",
+     "while (i < n_spans && span_start[i] == span_end[i]) {\n            anchor_row += span_groups[i];",
+     "while (i < n_spans && span_start[i] == span_end[i]) {"),
+    ("group mean divides by |G|+1", "double exact = sum / (double)(hi - lo);",
+     "double exact = sum / (double)(hi - lo + 1);"),
+    ("stored mean divides by |G|+1", "float stored = acc / (float)(hi - lo);",
+     "float stored = acc / (float)(hi - lo + 1);"),
+    ("bf16 rounds half up", "u += 0x7fffu + lsb;", "u += 0x8000u;"),
+    ("bf16 truncates", "u += 0x7fffu + lsb;", "u += 0u;"),
+    ("background position off by one", "pos[slot] = t;\n            slot_map[t] = slot;",
+     "pos[slot] = t + 1;\n            slot_map[t] = slot;"),
+    ("group position is its last token", "pos[slot] = (int32_t)lo;", "pos[slot] = (int32_t)(hi - 1);"),
+    ("ties go to the higher position", "return (x->pos > y->pos) - (x->pos < y->pos);",
+     "return (x->pos < y->pos) - (x->pos > y->pos);"),
+    ("lowest scores kept", "if (x->score > y->score)\n        return -1;\n    if (x->score < y->score)\n        return 1;",
+     "if (x->score > y->score)\n        return 1;\n    if (x->score < y->score)\n        return -1;"),
+    ("recent window rounded up", "floor((double)recent_frac * (double)budget)",
+     "ceil((double)recent_frac * (double)budget)"),
+    ("recent window one short", "for (int32_t j = n - M; j < n; ++j)\n        keep[j] = 1;",
+     "for (int32_t j = n - M + 1; j < n; ++j)\n        keep[j] = 1;"),
+    ("sinks one short", "for (int32_t j = 0; j < T; ++j)\n        keep[j] = 1;",
+     "for (int32_t j = 0; j < T - 1; ++j)\n        keep[j] = 1;"),
+    ("score not moved with its row", "score[w] = score[j];", "(void)0;"),
+    ("position not moved with its row", "pos[w] = pos[j];", "(void)0;"),
+    ("margin against the wrong runner-up", "*margin = c[N - 1].score - c[N].score;",
+     "*margin = c[N - 1].score - c[N + 1 < nc ? N + 1 : N].score;"),
+]
+
+
+def _caught(orc):
+    for pin in oracle_pins.ALL_PINS:
+        try:
+            pin(orc)
+        except (AssertionError, oracle.OracleError, ValueError, FloatingPointError):
+            return pin.__name__
+    return None
+
+
+@pytest.mark.parametrize("name,old,new", MUTATIONS, ids=[m[0] for m in MUTATIONS])
+def test_planted_mistake_is_caught(tmp_path, name, old, new):
+    with open(oracle.SOURCE) as f:
+        src = f.read()
+    assert old in src, f"mutation anchor for '{name}' not found in the oracle source"
+    mutated = tmp_path / "mutant.c"
+    mutated.write_text(src.replace(old, new))
+    lib = oracle.build(force=True, src=str(mutated), out=str(tmp_path / "libmutant.so"))
+    by = _caught(oracle.Oracle(lib))
+    assert by is not None, f"no pin catches the planted mistake: {name}"
+    print(f"{name}: caught by {by}")
