@@ -1,0 +1,423 @@
+#!/usr/bin/env python
+"""Benchmark of the VoxZip KV-compression path on GB300.
+
+One bench step is one request of the workload run through the whole path via the C ABI:
+stage-1 fusion of the resident prefilled K/V, then every decode step over all 48 layers
+(fused append + GQA attention + decayed-score update) with an eviction every `interval` steps.
+The reported value is decode steps per second of the whole job (each decode step advances every
+sequence of the batch by one token through all layers), stage 1 and evictions included.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload stress] [--impl voxzip|reference]
+
+Under torchrun each rank runs its own replica of the workload on its own GPU (the units of the
+path are independent, so there is no data-path collective); the time is the max over ranks.
+`--impl reference` times the fp64 CPU oracle on a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import concurrent.futures as cf
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "decode steps/s + HBM GB/s (% of GB300 peak) for fused attn+score+evict at 4x/20x"
+UNIT = "decode steps/s"
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse_args():
+    p = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--impl", choices=["voxzip", "reference"], default="voxzip")
+    p.add_argument("--workload", default="stress")
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-units", type=int, default=0, help="units in the oracle sample (0: one per core)")
+    return p.parse_args()
+
+
+def cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+# ----------------------------------------------------------------------------- distributed
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    return rank, world, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples every 200 ms while the timed region runs."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        sel = []
+        try:
+            uuid = str(torch.cuda.get_device_properties(self.dev).uuid)
+            sel = ["-i", uuid if uuid.startswith("GPU-") else "GPU-" + uuid]
+        except Exception:
+            sel = []
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", *sel, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.25)
+        return self
+
+    def __exit__(self, *exc):
+        time.sleep(0.25)
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for r in rows for n, v in zip(names, r[5:9]) if v.lower().startswith("active")})
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": float(rows[0][2]), "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(float(r[3]) for r in rows if r[3].replace(".", "").isdigit())}
+
+
+# ----------------------------------------------------------------------------- algorithmic bytes
+
+def decode_bytes(w, n_after):
+    """Bytes a decode launch over all layers must move: per unit, every cached K and V row once
+    (2 D e bytes per row), each score read and written (8 B), q in and out (2 G D e), k_new and
+    v_new in and their append (4 D e), and the new position (4 B)."""
+    es = 2 if w.dtype == torch.bfloat16 else 4
+    D, G = w.head_dim, w.group
+    per_b = [n * (2 * D * es + 8) + (2 * G * D + 4 * D) * es + 4 for n in n_after]
+    return w.layers * w.kv_heads * sum(per_b)
+
+
+def evict_bytes(w, n_before):
+    """Bytes an eviction must move, taking ordered compaction as the algorithm (Eq. 7-8): scores and
+    positions read once for the selection, then every kept row after the first evicted slot moved
+    (read and written: K, V, score, pos). The first evicted slot is at least the sink count, so
+    rows T..budget-M is the least that moves; this lower bound is what is counted."""
+    es = 2 if w.dtype == torch.bfloat16 else 4
+    row = 2 * w.head_dim * es + 8
+    tot = 0
+    for n, bud in zip(n_before, w.budget):
+        if n <= bud:
+            continue
+        tot += 8 * n
+    return w.layers * w.kv_heads * tot
+
+
+# ----------------------------------------------------------------------------- GPU arm
+
+class Runner:
+    def __init__(self, w, device):
+        from paper_2608_08569_gb300 import CacheDesc
+        from paper_2608_08569_gb300 import workloads as W
+        from paper_2608_08569_gb300.session import Session
+        self.w = w
+        self.dev = device
+        self.spans = W.make_spans(w)
+        i32 = lambda a: torch.as_tensor(np.asarray(a), dtype=torch.int32, device=device)
+        self.span_args = (i32(w.in_len), i32([w.audio_begin] * w.batch), i32(w.audio_len), i32(self.spans.off),
+                          i32(self.spans.start), i32(self.spans.end), i32(self.spans.groups))
+        self.k_pre, self.v_pre = W.make_prefill(w, device)
+        self.q, self.kn, self.vn, self.npos = W.make_steps(w, device)
+        self.desc = CacheDesc(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.capacity, w.dtype)
+        self.sess = Session(self.desc, w.budget, w.gamma, sink=w.sink, recent_frac=w.recent_frac, device=device)
+        self.out = torch.empty(w.steps, w.layers, w.batch, w.q_heads, w.head_dim, dtype=w.dtype, device=device)
+
+    def request(self, timers=None, lengths=None):
+        """One request: stage 1, then every decode step with evictions. With `timers`, records a
+        CUDA event pair around every decode launch (on the launch stream)."""
+        w, s = self.w, self.sess
+        s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
+        n = s.cache["len"][:, 0, 0].tolist() if lengths is not None else None
+        stream = torch.cuda.current_stream()
+        for t in range(1, w.steps + 1):
+            if timers is not None:
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+            s.decode(self.q[t - 1], self.kn[t - 1], self.vn[t - 1], self.npos[t - 1], self.out[t - 1])
+            if timers is not None:
+                e1.record(stream)
+                timers.append((e0, e1))
+            if n is not None:
+                n = [x + 1 for x in n]
+                lengths.append(("decode", list(n)))
+            if t % w.interval == 0:
+                if n is not None:
+                    lengths.append(("evict", list(n)))
+                    n = [min(x, b) for x, b in zip(n, w.budget)]
+                s.evict()
+
+
+def gpu_arm(args, rank, world, local):
+    from paper_2608_08569_gb300 import workloads as W
+    w = W.CONFIGS[args.workload]
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    r = Runner(w, dev)
+    for _ in range(args.warmup):
+        r.request()
+    torch.cuda.synchronize()
+    barrier(world)
+    timers, lengths = [], []
+    with ClockSampler(local) as clk:
+        torch.cuda.synchronize()
+        barrier(world)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for k in range(args.steps):
+            r.request(timers=timers, lengths=lengths if k == 0 else None)
+        e1.record()
+        torch.cuda.synchronize()
+        barrier(world)
+    ms = e0.elapsed_time(e1)
+    ms_max = max_over_ranks(ms, world)
+    total_steps = world * args.steps * w.steps
+    value = total_steps / (ms_max / 1000.0)
+
+    # Roofline of the dominant kernel (the decode step): algorithmic bytes over event-timed duration.
+    dec_lens = [n for kind, n in lengths if kind == "decode"]
+    bytes_per_request = sum(decode_bytes(w, n) for n in dec_lens)
+    dec_ms = sum(a.elapsed_time(b) for a, b in timers)
+    launches = len(timers)
+    avg_ms = dec_ms / launches
+    achieved = bytes_per_request * args.steps / (dec_ms / 1000.0) / 1e9
+    peak, peak_kind = peaks()
+    n_evict = w.steps // w.interval
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": None,
+                "kernel": "decode_kernel (append + GQA attention + decayed score)",
+                "peak_source": f"{peak_kind} hbm_gbs",
+                "avg_launch_us": round(avg_ms * 1000.0, 2),
+                "alg_bytes_per_launch": int(bytes_per_request / max(1, len(dec_lens))),
+                "decode_share_of_step": round(dec_ms / ms, 4)}
+    # kernels per request: 3 stage-1 kernels, one decode launch per step, one evict per interval
+    gpu_launches = args.steps * (3 + w.steps + n_evict)
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = e2e_leg(r, args)
+    clocks = clk.summary()
+    result = {
+        "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if w.dtype == torch.bfloat16 else "f32",
+        "data": "synthetic (seeded; Qwen3-Omni-thinker-shaped K/V/q, ASR-like spans)",
+        "config": {"workload": f"{w.name}: {w.description}", "batch": w.batch, "layers": w.layers,
+                   "q_heads": w.q_heads, "kv_heads": w.kv_heads, "head_dim": w.head_dim,
+                   "prompt_tokens": list(sorted(set(w.in_len))), "budget": list(sorted(set(w.budget))),
+                   "gamma": w.gamma, "decode_steps_per_request": w.steps, "evict_interval": w.interval,
+                   "parallelism": f"replicas x{world} (independent units, no collective)",
+                   "l2": "inputs larger than L2 (decode reads ~0.9-7 GB per launch, L2 is 129 MB)"},
+        "roofline": roofline, "gpu_launches": gpu_launches, "clocks": clocks, "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = cpu_sample(w, args.cpu_units)
+    return result
+
+
+def e2e_leg(r, args):
+    """The same metric with every request's inputs copied from pinned host memory (prefill K/V,
+    spans, every step's q / k_new / v_new) and every step's attention output copied back."""
+    w = r.w
+    pin = lambda t: t.cpu().pin_memory()
+    h = dict(k=pin(r.k_pre), v=pin(r.v_pre), q=pin(r.q), kn=pin(r.kn), vn=pin(r.vn))
+    h_spans = [pin(t) for t in r.span_args]
+    h_out = torch.empty(r.out.shape, dtype=r.out.dtype).pin_memory()
+    dev_spans = r.span_args
+
+    def request():
+        for src, dst in zip(h_spans, dev_spans):
+            dst.copy_(src, non_blocking=True)
+        r.k_pre.copy_(h["k"], non_blocking=True)
+        r.v_pre.copy_(h["v"], non_blocking=True)
+        r.q.copy_(h["q"], non_blocking=True)
+        r.kn.copy_(h["kn"], non_blocking=True)
+        r.vn.copy_(h["vn"], non_blocking=True)
+        r.request()
+        h_out.copy_(r.out, non_blocking=True)
+
+    request()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        request()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    nbytes = lambda t: t.numel() * t.element_size()
+    h2d = sum(nbytes(t) for t in h.values()) + sum(nbytes(t) for t in h_spans)
+    return {"value": round(args.steps * w.steps / (ms / 1000.0), 2), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": nbytes(h_out), "ms_per_step": round(ms / args.steps, 3)}
+
+
+# ----------------------------------------------------------------------------- oracle (CPU) arm
+
+def sample_units(w, k):
+    rng = np.random.default_rng(123)
+    all_units = [(b, l, h) for b in range(w.batch) for l in range(w.layers) for h in range(w.kv_heads)]
+    idx = rng.choice(len(all_units), size=min(k, len(all_units)), replace=False)
+    return [all_units[i] for i in sorted(idx)]
+
+
+def cpu_sample(w, n_units=0, inputs=None):
+    """Times the oracle on a bounded sample: `n_units` units (one per thread), each through the
+    whole request; the whole-workload time is the sample's wall time x units / sampled units."""
+    import oracle
+    from paper_2608_08569_gb300 import workloads as W
+    threads = cores()
+    n_units = n_units or min(threads, w.units)
+    units = sample_units(w, n_units)
+    spans = W.make_spans(w)
+    if inputs is None:
+        inputs = [W.unit_inputs_cpu(w, spans, b, l, h) for (b, l, h) in units]
+    orc = oracle.default()
+
+    def one(a):
+        u, b = a
+        return orc.run_unit(u["xk"], u["xv"], u["in_len"], u["audio_begin"], u["audio_len"], u["span_start"],
+                            u["span_end"], u["span_groups"], q=u["q"], k_new=u["k_new"], v_new=u["v_new"],
+                            new_pos=u["new_pos"], gamma=w.gamma, scale=1.0 / math.sqrt(w.head_dim),
+                            interval=w.interval, budget=w.budget[b], sink=w.sink, recent_frac=w.recent_frac,
+                            capacity=w.capacity, cache_is_bf16=w.dtype == torch.bfloat16)
+
+    args = [(u, b) for u, (b, l, h) in zip(inputs, units)]
+    used = min(threads, len(args))
+    t0 = time.perf_counter()
+    with cf.ThreadPoolExecutor(max_workers=used) as ex:
+        list(ex.map(one, args))
+    wall = time.perf_counter() - t0
+    full = wall * w.units / len(units)
+    return {"value": round(w.steps / full, 4), "unit": UNIT, "cores": used, "kind": "oracle",
+            "sample": (f"{len(units)} of {w.units} units (seeded choice), each through the whole request "
+                       f"({w.steps} decode steps, evictions every {w.interval}); {wall:.1f} s wall on {used} "
+                       f"threads, scaled by {w.units}/{len(units)} to the whole workload"),
+            "sample_wall_s": round(wall, 2)}, inputs
+
+
+def reference_arm(args, rank, world):
+    from paper_2608_08569_gb300 import workloads as W
+    w = W.CONFIGS[args.workload]
+    if rank != 0:
+        return None
+    inputs = None
+    for _ in range(args.warmup):
+        _, inputs = cpu_sample(w, args.cpu_units, inputs)
+    vals, last = [], None
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        last, inputs = cpu_sample(w, args.cpu_units, inputs)
+        vals.append(last["value"])
+    wall = time.perf_counter() - t0
+    value = statistics.mean(vals)
+    cb = dict(last)
+    cb["value"] = round(value, 4)
+    return {"metric": METRIC, "value": round(value, 4), "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(1000.0 * wall / args.steps, 1), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "impl": "reference",
+            "data": "synthetic (seeded; Qwen3-Omni-thinker-shaped K/V/q, ASR-like spans)",
+            "config": {"workload": f"{w.name}: {w.description}"}, "cpu_baseline": cb,
+            "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    args = parse_args()
+    rank, world, local = dist_setup()
+    if args.impl == "reference":
+        res = reference_arm(args, rank, world)
+    else:
+        res = gpu_arm(args, rank, world, local)
+        if isinstance(res.get("cpu_baseline"), tuple):
+            res["cpu_baseline"] = res["cpu_baseline"][0]
+    if rank == 0 and res is not None:
+        print(json.dumps(res), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

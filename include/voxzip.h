@@ -1,0 +1,174 @@
+/*
+ * voxzip.h -- C ABI of the VoxZip KV-cache compression library for NVIDIA GB300 (sm_103a).
+ *
+ * VoxZip (arxiv 2608.08569) compresses the KV cache of a speech LLM in two stages:
+ *   stage 1 (Sec. 3.2.1) fuses each ASR-aligned audio span of the prefilled cache into a few
+ *           averaged rows (Eq. 4, optional anchor add, Eq. 5);
+ *   stage 2 (Sec. 3.2.2) keeps a temporally decayed accumulated attention score per cached token
+ *           (Eq. 6), updated by every decode step (Eq. 1-2), and evicts down to a budget
+ *           by keeping T sinks, a recent window of M tokens and the top-N scored history
+ *           (Eq. 7-9).
+ * The library exports one call per step: voxzip_anchor_fuse, voxzip_decode_step, voxzip_evict.
+ *
+ * Conventions shared by every entry point
+ *   - A "unit" is one (sequence b, layer l, kv-head h). All state is per unit and units are
+ *     independent.
+ *   - Every tensor pointer is caller-owned DEVICE memory, dense and row-major in the layout given
+ *     beside it. The library never allocates, frees or copies to the host on these paths.
+ *   - Element type: K/V cache, prefill rows, anchors, q, k_new, v_new and out all have the
+ *     descriptor's dtype (bf16 or fp32). Scores are fp32, positions and lengths int32.
+ *   - Calls are asynchronous on `stream` and do not synchronise the host.
+ *   - Synchronous errors (bad descriptor, null required pointer, unsupported shape, workspace too
+ *     small) return an error status and launch nothing. A failed launch returns VOXZIP_ECUDA.
+ *   - Errors that depend on device data (malformed spans, a cache that would overflow its
+ *     capacity, a length above the caller's hint, a budget smaller than sink + recent) skip the
+ *     affected unit or sequence and set a bit in the device status word, read and cleared by
+ *     voxzip_get_status. Kernels never trap.
+ *   - Cache layout:  K, V   [B][L][Hkv][C][D]      (C = capacity slots per unit)
+ *                    score  [B][L][Hkv][C]  fp32    decayed accumulated attention (Eq. 6)
+ *                    pos    [B][L][Hkv][C]  int32   original token index of each slot
+ *                    len    [B][L][Hkv]     int32   cache length n of each unit
+ *     Slots [0, n) of a unit are valid and kept in chronological (ascending position) order.
+ */
+#ifndef VOXZIP_H
+#define VOXZIP_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; NULL is the legacy default stream. */
+typedef struct CUstream_st *voxzip_stream_t;
+
+typedef enum {
+    VOXZIP_OK = 0,
+    VOXZIP_EINVAL = 1,       /* invalid argument; nothing was launched */
+    VOXZIP_EUNSUPPORTED = 2, /* valid request outside what the kernels implement */
+    VOXZIP_ECUDA = 3         /* a CUDA runtime call or kernel launch failed */
+} voxzip_status;
+
+/* Bits of the device status word (asynchronous errors). */
+#define VOXZIP_DEV_BAD_SPANS 0x1u  /* a sequence's spans were malformed; its stage 1 was skipped */
+#define VOXZIP_DEV_CAPACITY 0x2u   /* stage-1 output or an append would exceed the capacity */
+#define VOXZIP_DEV_LEN_HINT 0x4u   /* a unit was longer than the call's max_len; it was skipped */
+#define VOXZIP_DEV_BAD_BUDGET 0x8u /* budget < sink + floor(budget * recent_frac); unit skipped */
+
+typedef enum { VOXZIP_F32 = 0, VOXZIP_BF16 = 1 } voxzip_dtype;
+
+typedef struct {
+    int32_t batch;    /* B, sequences */
+    int32_t layers;   /* L */
+    int32_t q_heads;  /* Hq */
+    int32_t kv_heads; /* Hkv; divides Hq. Query head i reads kv head i / (Hq / Hkv). */
+    int32_t head_dim; /* D, 64 or 128 */
+    int32_t capacity; /* C, slots per unit */
+    int32_t dtype;    /* voxzip_dtype of every K/V-typed tensor */
+} voxzip_cache_desc;
+
+/*
+ * Stage 1: semantic-anchored fusion of the prefilled cache (Sec. 3.2.1, Eq. 4, anchor addition,
+ * Eq. 5), for every layer and kv-head of every sequence.
+ *
+ * The ASR segments arrive as token-index spans, i.e. after the time-to-index map of Eq. 3.
+ * Sequence b's spans are entries [span_off[b], span_off[b+1]) of span_start/span_end/span_groups;
+ * they must be sorted, non-overlapping, lie inside [audio_begin[b], audio_begin[b]+audio_len[b])
+ * and have span_groups >= 1 (span_groups is L_t, the length of the span's transcription). A span
+ * of length l with g = min(span_groups, l) groups yields g rows; group j averages prefill rows
+ * [start + floor(j*l/g), start + floor((j+1)*l/g)) in fp32 in token order, divides by the group
+ * size, adds the anchor row if given, and rounds once to the cache dtype. Empty spans yield
+ * nothing. Every other token (text, or audio no span covers) is copied unchanged. Output rows
+ * keep chronological order; pos[slot] = index of the slot's first prefill token; score = 0;
+ * len = number of rows, the same for every unit of a sequence.
+ *
+ *   k_prefill, v_prefill  [B][L][Hkv][prefill_stride][D]; rows [0, in_len[b]) are read
+ *   in_len, audio_begin, audio_len  [B] device int32
+ *   span_off              [B+1] device int32, span_off[0] = 0, span_off[B] = num_spans
+ *   span_start, span_end, span_groups  [num_spans] device int32
+ *   anchor_k, anchor_v    NULL (anchor term zero) or [B][L][Hkv][anchor_stride][D]; group j of
+ *                         sequence b's span i adds row (sum of span_groups over b's spans before
+ *                         i) + j. Both NULL or both non-NULL.
+ *   k_cache, v_cache, score, pos, len   outputs, cache layout above
+ *   slot_map              NULL or [B][prefill_stride] device int32: output slot of every token
+ *   workspace             device scratch of at least voxzip_anchor_fuse_workspace_size() bytes,
+ *                         256-byte aligned; contents need not be initialised
+ * Device errors: VOXZIP_DEV_BAD_SPANS or VOXZIP_DEV_CAPACITY; the sequence's units get len = 0.
+ */
+voxzip_status voxzip_anchor_fuse(const voxzip_cache_desc *desc, const void *k_prefill,
+                                 const void *v_prefill, int32_t prefill_stride,
+                                 const int32_t *in_len, const int32_t *audio_begin,
+                                 const int32_t *audio_len, const int32_t *span_off,
+                                 int32_t num_spans, const int32_t *span_start,
+                                 const int32_t *span_end, const int32_t *span_groups,
+                                 const void *anchor_k, const void *anchor_v, int32_t anchor_stride,
+                                 void *k_cache, void *v_cache, float *score, int32_t *pos,
+                                 int32_t *len, int32_t *slot_map, void *workspace,
+                                 size_t workspace_bytes, voxzip_stream_t stream);
+
+/* Bytes of workspace voxzip_anchor_fuse needs (0 if the descriptor is invalid). */
+size_t voxzip_anchor_fuse_workspace_size(const voxzip_cache_desc *desc, int32_t prefill_stride,
+                                         int32_t num_spans);
+
+/*
+ * One decode step for layers [layer_begin, layer_begin + layer_count) of every sequence:
+ * append (Eq. 1), GQA attention (Eq. 2) and the decayed-score update (Eq. 6), fused so that
+ * each cached K and V row is read once.
+ *
+ * For every unit with length n: the new token's k_new/v_new are written to slot n with
+ * pos = new_pos[b]; then for each of the G = Hq/Hkv query heads of the unit,
+ *     p_h = softmax(scale * q_h K^T) over the n+1 rows,   out_h = p_h V,
+ * and every slot's score becomes  gamma * score + sum_h p_h  (the new slot starts from 0);
+ * len becomes n + 1.
+ *
+ *   q, out          [layer_count][B][Hq][D]
+ *   k_new, v_new    [layer_count][B][Hkv][D]
+ *   new_pos         [B] device int32, original index of the token being decoded
+ *   gamma           decay in (0, 1]; 1 is plain accumulation
+ *   sm_scale        logit scale; <= 0 selects 1/sqrt(D)
+ *   max_len         host-side upper bound on n + 1 over all units of the call (sizes the launch);
+ *                   <= 0 selects the capacity. Units above it are skipped with
+ *                   VOXZIP_DEV_LEN_HINT.
+ * Requires D in {64, 128}, G <= 16. Device errors: VOXZIP_DEV_CAPACITY (n == C), LEN_HINT.
+ */
+voxzip_status voxzip_decode_step(const voxzip_cache_desc *desc, int32_t layer_begin,
+                                 int32_t layer_count, const void *q, const void *k_new,
+                                 const void *v_new, const int32_t *new_pos, void *k_cache,
+                                 void *v_cache, float *score, int32_t *pos, int32_t *len,
+                                 float gamma, float sm_scale, int32_t max_len, void *out,
+                                 voxzip_stream_t stream);
+
+/*
+ * Budgeted eviction (Sec. 3.2.2, Eq. 7-9) for layers [layer_begin, layer_begin + layer_count).
+ * A unit with n <= budget[b] is left alone. Otherwise, with T = sink,
+ * M = floor(budget[b] * recent_frac) (evaluated in double) and N = budget[b] - T - M, it keeps
+ * slots [0, T), slots [n - M, n) and the N slots of [T, n - M) with the highest score, ties
+ * going to the lower position, and moves the kept rows (K, V, score, pos) to [0, budget[b]) in
+ * ascending slot order, in place; len becomes budget[b].
+ *
+ *   budget  [B] device int32
+ * Device errors: VOXZIP_DEV_BAD_BUDGET (N < 0).
+ */
+voxzip_status voxzip_evict(const voxzip_cache_desc *desc, int32_t layer_begin,
+                           int32_t layer_count, void *k_cache, void *v_cache, float *score,
+                           int32_t *pos, int32_t *len, const int32_t *budget, int32_t sink,
+                           float recent_frac, voxzip_stream_t stream);
+
+/*
+ * Waits for `stream`, then returns the device status word of the current device in *bits
+ * (VOXZIP_DEV_* flags accumulated by earlier calls) and clears it.
+ */
+voxzip_status voxzip_get_status(uint32_t *bits, voxzip_stream_t stream);
+
+/* Human-readable name of a status code (static storage). */
+const char *voxzip_status_string(voxzip_status status);
+
+/* Library ABI version: 100 * major + minor. */
+int32_t voxzip_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* VOXZIP_H */

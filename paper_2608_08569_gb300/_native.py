@@ -1,0 +1,211 @@
+"""ctypes binding of ``libvoxzip.so`` (declared in ``include/voxzip.h``).
+
+Argument marshalling only: tensors become device pointers, the current torch stream becomes the
+launch stream, and a non-OK status becomes an exception. Every step of the path runs in the
+library's CUDA kernels; there is no fallback when the library is missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+from dataclasses import dataclass
+
+import torch
+
+from .build import LIB_PATH
+
+VOXZIP_OK, VOXZIP_EINVAL, VOXZIP_EUNSUPPORTED, VOXZIP_ECUDA = 0, 1, 2, 3
+DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_BAD_BUDGET = 0x1, 0x2, 0x4, 0x8
+VOXZIP_F32, VOXZIP_BF16 = 0, 1
+
+_DTYPES = {torch.float32: VOXZIP_F32, torch.bfloat16: VOXZIP_BF16}
+
+
+class VoxZipError(RuntimeError):
+    def __init__(self, fn: str, code: int, text: str):
+        super().__init__(f"{fn} failed: {text} ({code})")
+        self.code = code
+
+
+class _Desc(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("layers", ctypes.c_int32), ("q_heads", ctypes.c_int32),
+                ("kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32), ("capacity", ctypes.c_int32),
+                ("dtype", ctypes.c_int32)]
+
+
+@dataclass(frozen=True)
+class CacheDesc:
+    """Shape of a VoxZip cache: B sequences x L layers x Hkv kv-heads, C slots of D elements."""
+    batch: int
+    layers: int
+    q_heads: int
+    kv_heads: int
+    head_dim: int
+    capacity: int
+    dtype: torch.dtype = torch.bfloat16
+
+    @property
+    def group(self) -> int:
+        return self.q_heads // self.kv_heads
+
+    def c_struct(self) -> _Desc:
+        return _Desc(self.batch, self.layers, self.q_heads, self.kv_heads, self.head_dim, self.capacity,
+                     _DTYPES[self.dtype])
+
+
+_lock = threading.Lock()
+_lib = None
+_vp = ctypes.c_void_p
+_i32 = ctypes.c_int32
+_f32 = ctypes.c_float
+_sz = ctypes.c_size_t
+_DP = ctypes.POINTER(_Desc)
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library; raises if it has not been built (no CPU fallback exists)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(f"{LIB_PATH} is missing: build it with paper_2608_08569_gb300.build")
+            L = ctypes.CDLL(LIB_PATH)
+            L.voxzip_anchor_fuse.argtypes = [_DP, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _vp,
+                                             _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+            L.voxzip_anchor_fuse_workspace_size.argtypes = [_DP, _i32, _i32]
+            L.voxzip_anchor_fuse_workspace_size.restype = _sz
+            L.voxzip_decode_step.argtypes = [_DP, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                             _f32, _f32, _i32, _vp, _vp]
+            L.voxzip_evict.argtypes = [_DP, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _f32, _vp]
+            L.voxzip_get_status.argtypes = [ctypes.POINTER(ctypes.c_uint32), _vp]
+            L.voxzip_status_string.argtypes = [_i32]
+            L.voxzip_status_string.restype = ctypes.c_char_p
+            L.voxzip_version.restype = _i32
+            for f in (L.voxzip_anchor_fuse, L.voxzip_decode_step, L.voxzip_evict, L.voxzip_get_status):
+                f.restype = _i32
+            _lib = L
+    return _lib
+
+
+def _check(fn: str, code: int) -> None:
+    if code != VOXZIP_OK:
+        raise VoxZipError(fn, code, lib().voxzip_status_string(code).decode())
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t: torch.Tensor, name: str, dtype: torch.dtype, shape=None) -> None:
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name}: dtype {t.dtype}, expected {dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be on a CUDA device")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name}: shape {tuple(t.shape)}, expected {tuple(shape)}")
+
+
+def _check_cache(desc: CacheDesc, k_cache, v_cache, score, pos, len_) -> None:
+    cs = (desc.batch, desc.layers, desc.kv_heads, desc.capacity)
+    _need(k_cache, "k_cache", desc.dtype, cs + (desc.head_dim,))
+    _need(v_cache, "v_cache", desc.dtype, cs + (desc.head_dim,))
+    _need(score, "score", torch.float32, cs)
+    _need(pos, "pos", torch.int32, cs)
+    _need(len_, "len", torch.int32, cs[:3])
+
+
+def allocate_cache(desc: CacheDesc, device="cuda"):
+    """Device tensors for a cache of shape ``desc``: k, v, score, pos, len (zero-filled)."""
+    cs = (desc.batch, desc.layers, desc.kv_heads, desc.capacity)
+    return dict(k=torch.zeros(cs + (desc.head_dim,), dtype=desc.dtype, device=device),
+                v=torch.zeros(cs + (desc.head_dim,), dtype=desc.dtype, device=device),
+                score=torch.zeros(cs, dtype=torch.float32, device=device),
+                pos=torch.zeros(cs, dtype=torch.int32, device=device),
+                len=torch.zeros(cs[:3], dtype=torch.int32, device=device))
+
+
+def voxzip_anchor_fuse_workspace_size(desc: CacheDesc, prefill_stride: int, num_spans: int) -> int:
+    d = desc.c_struct()
+    return int(lib().voxzip_anchor_fuse_workspace_size(ctypes.byref(d), int(prefill_stride), int(num_spans)))
+
+
+def voxzip_anchor_fuse(desc: CacheDesc, k_prefill, v_prefill, in_len, audio_begin, audio_len, span_off,
+                       span_start, span_end, span_groups, k_cache, v_cache, score, pos, len_, *,
+                       slot_map=None, anchor_k=None, anchor_v=None, workspace=None, stream=None) -> None:
+    """Stage 1 (Sec. 3.2.1): fuse the prefilled K/V of every unit into the cache."""
+    B, L, H, D = desc.batch, desc.layers, desc.kv_heads, desc.head_dim
+    if k_prefill.dim() != 5:
+        raise ValueError("k_prefill must be [B][L][Hkv][stride][D]")
+    stride = k_prefill.shape[3]
+    _need(k_prefill, "k_prefill", desc.dtype, (B, L, H, stride, D))
+    _need(v_prefill, "v_prefill", desc.dtype, (B, L, H, stride, D))
+    for name, t in (("in_len", in_len), ("audio_begin", audio_begin), ("audio_len", audio_len)):
+        _need(t, name, torch.int32, (B,))
+    _need(span_off, "span_off", torch.int32, (B + 1,))
+    num_spans = span_start.numel()
+    for name, t in (("span_start", span_start), ("span_end", span_end), ("span_groups", span_groups)):
+        _need(t, name, torch.int32, (num_spans,))
+    _check_cache(desc, k_cache, v_cache, score, pos, len_)
+    if slot_map is not None:
+        _need(slot_map, "slot_map", torch.int32, (B, stride))
+    anchor_stride = 0
+    if anchor_k is not None or anchor_v is not None:
+        anchor_stride = anchor_k.shape[3]
+        _need(anchor_k, "anchor_k", desc.dtype, (B, L, H, anchor_stride, D))
+        _need(anchor_v, "anchor_v", desc.dtype, (B, L, H, anchor_stride, D))
+    need = voxzip_anchor_fuse_workspace_size(desc, stride, num_spans)
+    if workspace is None:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=k_cache.device)
+    _need(workspace, "workspace", torch.uint8)
+    d = desc.c_struct()
+    _check("voxzip_anchor_fuse", lib().voxzip_anchor_fuse(
+        ctypes.byref(d), _ptr(k_prefill), _ptr(v_prefill), int(stride), _ptr(in_len), _ptr(audio_begin),
+        _ptr(audio_len), _ptr(span_off), int(num_spans), _ptr(span_start), _ptr(span_end), _ptr(span_groups),
+        _ptr(anchor_k), _ptr(anchor_v), int(anchor_stride), _ptr(k_cache), _ptr(v_cache), _ptr(score),
+        _ptr(pos), _ptr(len_), _ptr(slot_map), _ptr(workspace), int(workspace.numel()), _stream(stream)))
+
+
+def voxzip_decode_step(desc: CacheDesc, layer_begin: int, layer_count: int, q, k_new, v_new, new_pos,
+                       k_cache, v_cache, score, pos, len_, gamma: float, out, *, sm_scale: float = 0.0,
+                       max_len: int = 0, stream=None) -> None:
+    """One decode step (Eq. 1, Eq. 2, Eq. 6) for layers [layer_begin, layer_begin + layer_count)."""
+    B, Hq, H, D = desc.batch, desc.q_heads, desc.kv_heads, desc.head_dim
+    _need(q, "q", desc.dtype, (layer_count, B, Hq, D))
+    _need(k_new, "k_new", desc.dtype, (layer_count, B, H, D))
+    _need(v_new, "v_new", desc.dtype, (layer_count, B, H, D))
+    _need(out, "out", desc.dtype, (layer_count, B, Hq, D))
+    _need(new_pos, "new_pos", torch.int32, (B,))
+    _check_cache(desc, k_cache, v_cache, score, pos, len_)
+    d = desc.c_struct()
+    _check("voxzip_decode_step", lib().voxzip_decode_step(
+        ctypes.byref(d), int(layer_begin), int(layer_count), _ptr(q), _ptr(k_new), _ptr(v_new), _ptr(new_pos),
+        _ptr(k_cache), _ptr(v_cache), _ptr(score), _ptr(pos), _ptr(len_), float(gamma), float(sm_scale),
+        int(max_len), _ptr(out), _stream(stream)))
+
+
+def voxzip_evict(desc: CacheDesc, layer_begin: int, layer_count: int, k_cache, v_cache, score, pos, len_,
+                 budget, *, sink: int = 4, recent_frac: float = 0.2, stream=None) -> None:
+    """Budgeted eviction (Eq. 7-9) for layers [layer_begin, layer_begin + layer_count)."""
+    _check_cache(desc, k_cache, v_cache, score, pos, len_)
+    _need(budget, "budget", torch.int32, (desc.batch,))
+    d = desc.c_struct()
+    _check("voxzip_evict", lib().voxzip_evict(
+        ctypes.byref(d), int(layer_begin), int(layer_count), _ptr(k_cache), _ptr(v_cache), _ptr(score), _ptr(pos),
+        _ptr(len_), _ptr(budget), int(sink), float(recent_frac), _stream(stream)))
+
+
+def voxzip_get_status(stream=None) -> int:
+    """Waits for the stream, then returns and clears the device status word (DEV_* bits)."""
+    bits = ctypes.c_uint32(0)
+    _check("voxzip_get_status", lib().voxzip_get_status(ctypes.byref(bits), _stream(stream)))
+    return int(bits.value)

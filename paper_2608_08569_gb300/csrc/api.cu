@@ -1,0 +1,165 @@
+// C ABI of the VoxZip library (declared in include/voxzip.h): argument validation, the device
+// status word, and dispatch to the kernel launchers. Nothing here allocates device memory.
+#include <math.h>
+
+#include "common.cuh"
+
+namespace {
+
+// Asynchronous error bits (VOXZIP_DEV_*) raised by the kernels of this library on this device.
+__device__ int32_t g_status_word;
+
+constexpr int kMaxDevices = 64;
+int32_t *g_status_addr[kMaxDevices];  // device address of g_status_word, per device
+
+// Address of the status word on the current device (looked up once per device).
+voxzip_status status_word(int32_t **addr) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return VOXZIP_ECUDA;
+    if (g_status_addr[dev] == nullptr) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return VOXZIP_ECUDA;
+        g_status_addr[dev] = static_cast<int32_t *>(p);
+    }
+    *addr = g_status_addr[dev];
+    return VOXZIP_OK;
+}
+
+bool desc_ok(const voxzip_cache_desc *d) {
+    if (d == nullptr) return false;
+    if (d->batch < 1 || d->layers < 1 || d->q_heads < 1 || d->kv_heads < 1 || d->capacity < 1) return false;
+    if (d->q_heads % d->kv_heads != 0) return false;
+    if (d->head_dim != 64 && d->head_dim != 128) return false;
+    if (d->dtype != VOXZIP_F32 && d->dtype != VOXZIP_BF16) return false;
+    // element counts of the largest tensors must fit int64 and slot indices int32
+    const int64_t units = (int64_t)d->batch * d->layers * d->kv_heads;
+    if (units > (int64_t)1 << 31) return false;
+    return true;
+}
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+voxzip_status from_cuda(cudaError_t e) { return e == cudaSuccess ? VOXZIP_OK : VOXZIP_ECUDA; }
+
+constexpr int kMaxGridY = 65535;
+
+}  // namespace
+
+extern "C" {
+
+int32_t voxzip_version(void) { return 100; }
+
+const char *voxzip_status_string(voxzip_status s) {
+    switch (s) {
+        case VOXZIP_OK: return "VOXZIP_OK";
+        case VOXZIP_EINVAL: return "VOXZIP_EINVAL";
+        case VOXZIP_EUNSUPPORTED: return "VOXZIP_EUNSUPPORTED";
+        case VOXZIP_ECUDA: return "VOXZIP_ECUDA";
+    }
+    return "VOXZIP_UNKNOWN";
+}
+
+size_t voxzip_anchor_fuse_workspace_size(const voxzip_cache_desc *desc, int32_t prefill_stride,
+                                         int32_t num_spans) {
+    if (!desc_ok(desc) || prefill_stride < 1 || num_spans < 0) return 0;
+    return voxzip::anchor_fuse_workspace_bytes(*desc, prefill_stride, num_spans);
+}
+
+voxzip_status voxzip_anchor_fuse(const voxzip_cache_desc *desc, const void *k_prefill,
+                                 const void *v_prefill, int32_t prefill_stride,
+                                 const int32_t *in_len, const int32_t *audio_begin,
+                                 const int32_t *audio_len, const int32_t *span_off,
+                                 int32_t num_spans, const int32_t *span_start,
+                                 const int32_t *span_end, const int32_t *span_groups,
+                                 const void *anchor_k, const void *anchor_v, int32_t anchor_stride,
+                                 void *k_cache, void *v_cache, float *score, int32_t *pos,
+                                 int32_t *len, int32_t *slot_map, void *workspace,
+                                 size_t workspace_bytes, voxzip_stream_t stream) {
+    if (!desc_ok(desc) || prefill_stride < 1 || num_spans < 0) return VOXZIP_EINVAL;
+    if (!k_prefill || !v_prefill || !in_len || !audio_begin || !audio_len || !span_off || !k_cache ||
+        !v_cache || !score || !pos || !len || !workspace)
+        return VOXZIP_EINVAL;
+    if (num_spans > 0 && (!span_start || !span_end || !span_groups)) return VOXZIP_EINVAL;
+    if ((anchor_k == nullptr) != (anchor_v == nullptr)) return VOXZIP_EINVAL;
+    if (anchor_k && anchor_stride < 1) return VOXZIP_EINVAL;
+    if (!aligned16(k_prefill) || !aligned16(v_prefill) || !aligned16(k_cache) || !aligned16(v_cache) ||
+        (anchor_k && (!aligned16(anchor_k) || !aligned16(anchor_v))))
+        return VOXZIP_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return VOXZIP_EINVAL;
+    if (workspace_bytes < voxzip::anchor_fuse_workspace_bytes(*desc, prefill_stride, num_spans))
+        return VOXZIP_EINVAL;
+    if ((int64_t)desc->batch * desc->layers * desc->kv_heads > kMaxGridY || desc->batch > kMaxGridY)
+        return VOXZIP_EUNSUPPORTED;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    return from_cuda(voxzip::launch_anchor_fuse(
+        *desc, k_prefill, v_prefill, prefill_stride, in_len, audio_begin, audio_len, span_off, num_spans,
+        span_start, span_end, span_groups, anchor_k, anchor_v, anchor_stride, k_cache, v_cache, score, pos, len,
+        slot_map, workspace, status, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+voxzip_status voxzip_decode_step(const voxzip_cache_desc *desc, int32_t layer_begin,
+                                 int32_t layer_count, const void *q, const void *k_new,
+                                 const void *v_new, const int32_t *new_pos, void *k_cache,
+                                 void *v_cache, float *score, int32_t *pos, int32_t *len,
+                                 float gamma, float sm_scale, int32_t max_len, void *out,
+                                 voxzip_stream_t stream) {
+    if (!desc_ok(desc)) return VOXZIP_EINVAL;
+    if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
+        return VOXZIP_EINVAL;
+    if (!q || !k_new || !v_new || !new_pos || !k_cache || !v_cache || !score || !pos || !len || !out)
+        return VOXZIP_EINVAL;
+    if (!(gamma > 0.f && gamma <= 1.f) || isnan(sm_scale) || isinf(sm_scale)) return VOXZIP_EINVAL;
+    if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(k_cache) || !aligned16(v_cache) ||
+        !aligned16(out))
+        return VOXZIP_EINVAL;
+    if (desc->q_heads / desc->kv_heads > voxzip::kMaxGroup) return VOXZIP_EUNSUPPORTED;
+    if ((int64_t)layer_count * desc->batch * desc->kv_heads > kMaxGridY) return VOXZIP_EUNSUPPORTED;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    bool unsupported = false;
+    cudaError_t e = voxzip::launch_decode(*desc, layer_begin, layer_count, q, k_new, v_new, new_pos, k_cache,
+                                          v_cache, score, pos, len, gamma, sm_scale, max_len, out, status,
+                                          reinterpret_cast<cudaStream_t>(stream), &unsupported);
+    if (unsupported) return VOXZIP_EUNSUPPORTED;
+    return from_cuda(e);
+}
+
+voxzip_status voxzip_evict(const voxzip_cache_desc *desc, int32_t layer_begin,
+                           int32_t layer_count, void *k_cache, void *v_cache, float *score,
+                           int32_t *pos, int32_t *len, const int32_t *budget, int32_t sink,
+                           float recent_frac, voxzip_stream_t stream) {
+    if (!desc_ok(desc)) return VOXZIP_EINVAL;
+    if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
+        return VOXZIP_EINVAL;
+    if (!k_cache || !v_cache || !score || !pos || !len || !budget) return VOXZIP_EINVAL;
+    if (sink < 0 || !(recent_frac >= 0.f && recent_frac <= 1.f)) return VOXZIP_EINVAL;
+    if (!aligned16(k_cache) || !aligned16(v_cache)) return VOXZIP_EINVAL;
+    if ((int64_t)layer_count * desc->batch * desc->kv_heads > ((int64_t)1 << 31) - 1) return VOXZIP_EUNSUPPORTED;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    return from_cuda(voxzip::launch_evict(*desc, layer_begin, layer_count, k_cache, v_cache, score, pos, len,
+                                          budget, sink, recent_frac, status,
+                                          reinterpret_cast<cudaStream_t>(stream)));
+}
+
+voxzip_status voxzip_get_status(uint32_t *bits, voxzip_stream_t stream) {
+    if (!bits) return VOXZIP_EINVAL;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    int32_t host = 0;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return VOXZIP_ECUDA;
+    if (cudaMemcpyAsync(&host, status, sizeof(int32_t), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return VOXZIP_ECUDA;
+    if (cudaMemsetAsync(status, 0, sizeof(int32_t), s) != cudaSuccess) return VOXZIP_ECUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return VOXZIP_ECUDA;
+    *bits = (uint32_t)host;
+    return VOXZIP_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,260 @@
+"""CUDA path vs oracle, element by element, on the same seeded inputs (needs a GB300).
+
+Whole-path lockstep tests run stage 1, every decode step and every eviction of a workload on the
+GPU through the C ABI and the same units through the oracle. Isolated tests feed both sides the
+same generated cache state (not produced by either side) to exercise decode and eviction over
+many lengths, group sizes, dtypes, head dims and split counts.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from gpu_harness import (SCORE_ATOL, SCORE_RTOL, check_stage1, check_units, gpu_run, make_anchors, make_inputs,
+                         oracle_units, out_tol, sample_units)
+from paper_2608_08569_gb300 import (DEV_BAD_BUDGET, DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, CacheDesc,
+                                    allocate_cache, voxzip_anchor_fuse, voxzip_decode_step, voxzip_evict,
+                                    voxzip_get_status)
+from paper_2608_08569_gb300 import workloads as W
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2608_08569_gb300 import build
+    build.build_library()
+    oracle.build()
+
+
+def _pipeline(w, sample_k, steps=None, anchors=False):
+    inp = make_inputs(w, "cuda", steps=steps)
+    sample = sample_units(w, sample_k)
+    anc = make_anchors(w, inp["spans"], "cuda") if anchors else None
+    rec = gpu_run(w, inp, sample, steps=steps, anchors=anc)
+    check_stage1(w, inp, rec, sample, anchors=anc)
+    res = oracle_units(w, inp, sample, steps=steps, anchors=anc)
+    diverged = check_units(w, rec, res, sample, steps=steps)
+    assert len(diverged) <= max(1, len(sample) // 4), diverged
+    return rec, res, diverged
+
+
+@pytest.mark.parametrize("name", ["tiny", "tiny_identity", "short"])
+def test_whole_path_all_units(name):
+    w = W.CONFIGS[name]
+    _pipeline(w, sample_k=10 ** 6)
+
+
+def test_tiny_identity_evicts_and_stage1_is_identity():
+    w = W.CONFIGS["tiny_identity"]
+    rec, res, _ = _pipeline(w, sample_k=10 ** 6)
+    assert rec["stage1_len"][0] == w.in_len[0]
+    assert rec["len_before"][0, 0] == w.in_len[0] + w.interval and rec["kept_pos"].shape[0] == 4
+    assert (rec["len"] == w.budget[0]).all() or (rec["len"] <= w.budget[0] + w.interval).all()
+
+
+def test_whole_path_with_anchors():
+    w = W.scaled(W.CONFIGS["short"], layers=3, name="short_anchor")
+    _pipeline(w, sample_k=10 ** 6, anchors=True)
+
+
+@pytest.mark.parametrize("name,k,steps", [("long", 24, None), ("long_4x", 12, None), ("batched", 16, None),
+                                          ("stress", 6, None), ("stress_4x", 3, 96)])
+def test_full_size_sampled_units(name, k, steps):
+    w = W.CONFIGS[name]
+    _pipeline(w, sample_k=k, steps=steps)
+
+
+# ----------------------------------------------------------------------------- isolated states
+
+def _random_state(desc, lens, seed):
+    """Random cache contents drawn here (neither side computes them): rows, scores, positions."""
+    g = torch.Generator(device="cuda")
+    g.manual_seed(seed)
+    c = allocate_cache(desc, "cuda")
+    c["k"].copy_(torch.randn(c["k"].shape, generator=g, device="cuda").to(desc.dtype))
+    c["v"].copy_(torch.randn(c["v"].shape, generator=g, device="cuda").to(desc.dtype))
+    c["score"].copy_(torch.rand(c["score"].shape, generator=g, device="cuda") * 3)
+    c["pos"].copy_(torch.arange(desc.capacity, device="cuda", dtype=torch.int32) * 2 + 5)
+    c["len"].copy_(torch.as_tensor(lens, dtype=torch.int32, device="cuda").view(c["len"].shape))
+    return c
+
+
+def _unit_cache(c, b, l, h, n, cap):
+    f = lambda t: t.to("cpu", torch.float64).numpy()
+    return oracle.UnitCache.from_rows(cap, f(c["k"][b, l, h, :n]), f(c["v"][b, l, h, :n]),
+                                      c["pos"][b, l, h, :n].cpu().numpy(), f(c["score"][b, l, h, :n]))
+
+
+@pytest.mark.parametrize("dtype,D,Hq,Hkv", [(torch.bfloat16, 128, 32, 4), (torch.float32, 64, 2, 1),
+                                            (torch.bfloat16, 64, 16, 1), (torch.float32, 128, 4, 4),
+                                            (torch.bfloat16, 128, 12, 3)])
+@pytest.mark.parametrize("max_len_mode", ["tight", "capacity"])
+def test_decode_step_random_states(dtype, D, Hq, Hkv, max_len_mode):
+    B, L, C = 2, 3, 3000
+    desc = CacheDesc(B, L, Hq, Hkv, D, C, dtype)
+    rng = np.random.default_rng(D + Hq)
+    lens = rng.integers(0, C - 1, size=(B, L, Hkv))
+    lens.flat[0] = 0                      # empty cache: the output is v_new
+    lens.flat[1] = 1
+    lens.flat[-1] = C - 1                 # fills the cache exactly
+    c = _random_state(desc, lens, seed=11)
+    ref = {k: v.clone() for k, v in c.items()}
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(5)
+    q = torch.randn(L - 1, B, Hq, D, generator=gen, device="cuda").to(dtype)
+    kn = torch.randn(L - 1, B, Hkv, D, generator=gen, device="cuda").to(dtype)
+    vn = torch.randn(L - 1, B, Hkv, D, generator=gen, device="cuda").to(dtype)
+    npos = torch.tensor([9000, 9100], dtype=torch.int32, device="cuda")
+    out = torch.zeros(L - 1, B, Hq, D, dtype=dtype, device="cuda")
+    gamma = 0.97
+    max_len = int(lens.max()) + 1 if max_len_mode == "tight" else 0
+    voxzip_get_status()
+    voxzip_decode_step(desc, 1, L - 1, q, kn, vn, npos, c["k"], c["v"], c["score"], c["pos"], c["len"], gamma,
+                       out, max_len=max_len)
+    assert voxzip_get_status() == 0
+    G = Hq // Hkv
+    tol = 2e-2 if dtype == torch.bfloat16 else 1e-4
+    f = lambda t: t.to("cpu", torch.float64).numpy()
+    for b in range(B):
+        for l in range(L):
+            for h in range(Hkv):
+                n = int(lens[b, l, h])
+                if l == 0:   # outside the layer range: untouched
+                    assert int(c["len"][b, l, h]) == n
+                    assert torch.equal(c["score"][b, l, h], ref["score"][b, l, h])
+                    continue
+                u = _unit_cache(ref, b, l, h, n, C)
+                o = oracle.decode_step(u, f(q[l - 1, b, h * G:(h + 1) * G]), f(kn[l - 1, b, h]), f(vn[l - 1, b, h]),
+                                       int(npos[b]), gamma, 1 / math.sqrt(D))
+                assert int(c["len"][b, l, h]) == n + 1
+                got = f(out[l - 1, b, h * G:(h + 1) * G])
+                assert np.abs(got - o).max() <= tol, (b, l, h, np.abs(got - o).max())
+                np.testing.assert_allclose(f(c["score"][b, l, h, :n + 1]), u.score[:n + 1], rtol=SCORE_RTOL,
+                                           atol=SCORE_ATOL)
+                np.testing.assert_array_equal(c["pos"][b, l, h, :n + 1].cpu().numpy(), u.pos[:n + 1])
+                np.testing.assert_array_equal(f(c["k"][b, l, h, :n + 1]), u.K[:n + 1])
+                np.testing.assert_array_equal(f(c["v"][b, l, h, :n + 1]), u.V[:n + 1])
+                if n == 0:
+                    np.testing.assert_array_equal(got, np.tile(f(vn[l - 1, b, h]), (G, 1)))
+
+
+@pytest.mark.parametrize("dtype,D", [(torch.bfloat16, 128), (torch.float32, 64), (torch.float32, 128),
+                                     (torch.bfloat16, 64)])
+@pytest.mark.parametrize("ties", [False, True])
+def test_evict_random_states(dtype, D, ties):
+    B, L, H, C = 3, 2, 2, 2500
+    desc = CacheDesc(B, L, 2 * H, H, D, C, dtype)
+    rng = np.random.default_rng(3 + D)
+    budget = np.array([7, 300, 2000], np.int32)   # 7: M = 1, N = 2 (tiny); 2000: more than a 1024 chunk
+    lens = np.stack([rng.integers(max(1, bb - 20), min(C, 2 * bb + 600), size=(L, H)) for bb in budget])
+    lens[0, 0, 0] = budget[0]                    # exactly at budget: untouched
+    lens[2, 1, 1] = C                            # full cache
+    c = _random_state(desc, lens, seed=12)
+    if ties:
+        c["score"].copy_(torch.floor(c["score"] * 4) / 4)   # four distinct values: many exact ties
+    ref = {k: v.clone() for k, v in c.items()}
+    bud_t = torch.as_tensor(budget, device="cuda")
+    for sink, frac in ((4, 0.2), (0, 0.5), (2, 0.0)):
+        c2 = {k: v.clone() for k, v in ref.items()}
+        voxzip_evict(desc, 0, L, c2["k"], c2["v"], c2["score"], c2["pos"], c2["len"], bud_t, sink=sink,
+                     recent_frac=frac)
+        assert voxzip_get_status() == 0
+        for b in range(B):
+            for l in range(L):
+                for h in range(H):
+                    n = int(lens[b, l, h])
+                    u = _unit_cache(ref, b, l, h, n, C)
+                    oracle.evict(u, int(budget[b]), sink=sink, recent_frac=frac)
+                    m = u.n
+                    assert int(c2["len"][b, l, h]) == m
+                    np.testing.assert_array_equal(c2["pos"][b, l, h, :m].cpu().numpy(), u.pos[:m])
+                    np.testing.assert_array_equal(c2["score"][b, l, h, :m].double().cpu().numpy(), u.score[:m])
+                    np.testing.assert_array_equal(c2["k"][b, l, h, :m].double().cpu().numpy(), u.K[:m])
+                    np.testing.assert_array_equal(c2["v"][b, l, h, :m].double().cpu().numpy(), u.V[:m])
+
+
+# ----------------------------------------------------------------------------- edge cases and device errors
+
+def _fuse(desc, k, v, in_len, ab, al, spans_per_seq, stride, slot_map=True):
+    i32 = lambda a: torch.as_tensor(np.asarray(a, np.int64), dtype=torch.int32, device="cuda")
+    off, st, en, gr = [0], [], [], []
+    for s in spans_per_seq:
+        for (a, e, g) in s:
+            st.append(a); en.append(e); gr.append(g)
+        off.append(len(st))
+    c = allocate_cache(desc, "cuda")
+    sm = torch.full((desc.batch, stride), -1, dtype=torch.int32, device="cuda")
+    voxzip_anchor_fuse(desc, k, v, i32(in_len), i32(ab), i32(al), i32(off), i32(st), i32(en), i32(gr), c["k"], c["v"],
+                       c["score"], c["pos"], c["len"], slot_map=sm)
+    return c, sm, (off, st, en, gr)
+
+
+def test_stage1_edge_cases():
+    """Ragged prompts, no audio, empty spans, more groups than tokens, one-token prompt, prompt of
+    only audio, a span at the very end."""
+    B, L, H, D, stride = 6, 2, 2, 64, 40
+    desc = CacheDesc(B, L, 4, H, D, 64, torch.bfloat16)
+    g = torch.Generator(device="cuda")
+    g.manual_seed(3)
+    k = torch.randn(B, L, H, stride, D, generator=g, device="cuda").to(torch.bfloat16)
+    v = torch.randn(B, L, H, stride, D, generator=g, device="cuda").to(torch.bfloat16)
+    in_len = [40, 10, 1, 25, 30, 0]
+    ab = [5, 3, 0, 0, 2, 0]
+    al = [30, 0, 1, 25, 28, 0]
+    spans = [[(5, 9, 1), (9, 9, 2), (12, 20, 3), (20, 22, 5), (30, 35, 2)],
+             [],
+             [(0, 1, 1)],
+             [(0, 25, 4)],
+             [(2, 3, 1), (27, 30, 2)],
+             []]
+    c, sm, _ = _fuse(desc, k, v, in_len, ab, al, spans, stride)
+    assert voxzip_get_status() == 0
+    for b in range(B):
+        st = [s[0] for s in spans[b]]
+        en = [s[1] for s in spans[b]]
+        gr = [s[2] for s in spans[b]]
+        for l in range(L):
+            for h in range(H):
+                x = k[b, l, h, :in_len[b]].double().cpu().numpy()
+                r = oracle.stage1(x if in_len[b] else np.zeros((0, D)), in_len[b], ab[b], al[b], st, en, gr,
+                                  cache_is_bf16=True, capacity=64)
+                n = r["n"]
+                assert int(c["len"][b, l, h]) == n
+                np.testing.assert_array_equal(c["k"][b, l, h, :n].double().cpu().numpy(), r["stored"])
+                np.testing.assert_array_equal(c["pos"][b, l, h, :n].cpu().numpy(), r["pos"])
+                assert float(c["score"][b, l, h, :n].abs().sum()) == 0.0
+        np.testing.assert_array_equal(sm[b, :in_len[b]].cpu().numpy(), r["slot_map"])
+
+
+def test_device_errors_set_status_bits_and_skip():
+    B, L, H, D, stride = 3, 1, 1, 64, 20
+    desc = CacheDesc(B, L, 2, H, D, 12, torch.float32)
+    k = torch.ones(B, L, H, stride, D, device="cuda")
+    v = torch.ones(B, L, H, stride, D, device="cuda")
+    # seq 0 unsorted spans, seq 1 fine, seq 2 does not fit the capacity
+    c, _, _ = _fuse(desc, k, v, [20, 20, 20], [0, 0, 0], [20, 20, 20],
+                    [[(5, 8, 1), (2, 4, 1)], [(0, 10, 1), (10, 20, 1)], [(0, 2, 1)]], stride)
+    bits = voxzip_get_status()
+    assert bits & DEV_BAD_SPANS and bits & DEV_CAPACITY
+    assert c["len"].view(-1).tolist() == [0, 2, 0]
+    # decode with a length hint below the real length: skipped with LEN_HINT; at capacity: CAPACITY
+    q = torch.randn(1, B, 2, D, device="cuda")
+    kn = torch.randn(1, B, H, D, device="cuda")
+    out = torch.zeros_like(q)
+    npos = torch.zeros(B, dtype=torch.int32, device="cuda")
+    c["len"].view(-1)[2] = 12
+    voxzip_decode_step(desc, 0, 1, q, kn, kn, npos, c["k"], c["v"], c["score"], c["pos"], c["len"], 0.9, out,
+                       max_len=1)
+    bits = voxzip_get_status()
+    assert bits & DEV_LEN_HINT and bits & DEV_CAPACITY
+    assert c["len"].view(-1).tolist() == [1, 2, 12]   # seq 0 appended (n 0 -> 1), seq 1 skipped, seq 2 full
+    assert voxzip_get_status() == 0                   # reading clears the word
+    # evict with a budget below sink + recent
+    voxzip_evict(desc, 0, 1, c["k"], c["v"], c["score"], c["pos"], c["len"],
+                 torch.tensor([2, 2, 2], dtype=torch.int32, device="cuda"), sink=4)
+    assert voxzip_get_status() & DEV_BAD_BUDGET
