@@ -301,7 +301,17 @@ def e2e_leg(r, args):
     """The same metric with every request's inputs copied from pinned host memory (prefill K/V,
     spans, every step's q / k_new / v_new) and every step's attention output copied back."""
     w = r.w
-    pin = lambda t: t.cpu().pin_memory()
+    nbytes = lambda t: t.numel() * t.element_size()
+    need = sum(nbytes(t) for t in (r.k_pre, r.v_pre, r.q, r.kn, r.vn, r.out))
+    avail = host_mem_available()
+    if avail is not None and avail < 1.5 * need + (8 << 30):
+        return {"value": None, "unit": UNIT, "skipped": f"host memory: {avail >> 30} GiB available, "
+                                                        f"{need >> 30} GiB of pinned buffers needed"}
+
+    def pin(t):
+        h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        h.copy_(t)
+        return h
     h = dict(k=pin(r.k_pre), v=pin(r.v_pre), q=pin(r.q), kn=pin(r.kn), vn=pin(r.vn))
     h_spans = [pin(t) for t in r.span_args]
     h_out = torch.empty(r.out.shape, dtype=r.out.dtype).pin_memory()
@@ -328,10 +338,31 @@ def e2e_leg(r, args):
     e1.record()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
-    nbytes = lambda t: t.numel() * t.element_size()
     h2d = sum(nbytes(t) for t in h.values()) + sum(nbytes(t) for t in h_spans)
     return {"value": round(args.steps * w.steps / (ms / 1000.0), 2), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": nbytes(h_out), "ms_per_step": round(ms / args.steps, 3)}
+
+
+def host_mem_available():
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    avail = int(line.split()[1]) * 1024
+                    break
+            else:
+                return None
+    except OSError:
+        return None
+    for path in ("/sys/fs/cgroup/memory.max",):
+        try:
+            with open(path) as f:
+                lim = f.read().strip()
+            if lim != "max":
+                avail = min(avail, int(lim))
+        except (OSError, ValueError):
+            pass
+    return avail
 
 
 # ----------------------------------------------------------------------------- oracle (CPU) arm

@@ -55,6 +55,8 @@ typedef enum {
 #define VOXZIP_DEV_CAPACITY 0x2u   /* stage-1 output or an append would exceed the capacity */
 #define VOXZIP_DEV_LEN_HINT 0x4u   /* a unit was longer than the call's max_len; it was skipped */
 #define VOXZIP_DEV_BAD_BUDGET 0x8u /* budget < sink + floor(budget * recent_frac); unit skipped */
+#define VOXZIP_DEV_TIMEOUT 0x10u   /* a bounded wait inside a kernel gave up; outputs of that unit
+                                      are not valid (never expected; reported instead of hanging) */
 
 typedef enum { VOXZIP_F32 = 0, VOXZIP_BF16 = 1 } voxzip_dtype;
 

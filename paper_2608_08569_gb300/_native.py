@@ -16,7 +16,7 @@ import torch
 from .build import LIB_PATH
 
 VOXZIP_OK, VOXZIP_EINVAL, VOXZIP_EUNSUPPORTED, VOXZIP_ECUDA = 0, 1, 2, 3
-DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_BAD_BUDGET = 0x1, 0x2, 0x4, 0x8
+DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_BAD_BUDGET, DEV_TIMEOUT = 0x1, 0x2, 0x4, 0x8, 0x10
 VOXZIP_F32, VOXZIP_BF16 = 0, 1
 
 _DTYPES = {torch.float32: VOXZIP_F32, torch.bfloat16: VOXZIP_BF16}

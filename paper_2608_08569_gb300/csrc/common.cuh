@@ -86,6 +86,12 @@ cudaError_t launch_decode(const voxzip_cache_desc &d, int32_t layer_begin, int32
                           float gamma, float sm_scale, int32_t max_len, void *out, int32_t *status,
                           cudaStream_t stream, bool *unsupported);
 
+bool decode_mma_supported(const voxzip_cache_desc &d);
+cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, int32_t layer_count, const void *q,
+                              const void *k_new, const void *v_new, const int32_t *new_pos, void *k_cache,
+                              void *v_cache, float *score, int32_t *pos, int32_t *len, float gamma, float sm_scale,
+                              int32_t max_len, void *out, int32_t *status, cudaStream_t stream, bool *unsupported);
+
 cudaError_t launch_evict(const voxzip_cache_desc &d, int32_t layer_begin, int32_t layer_count,
                          void *k_cache, void *v_cache, float *score, int32_t *pos, int32_t *len,
                          const int32_t *budget, int32_t sink, float recent_frac, int32_t *status,

@@ -234,6 +234,13 @@ cudaError_t launch_decode(const voxzip_cache_desc &d, int32_t layer_begin, int32
                           float gamma, float sm_scale, int32_t max_len, void *out, int32_t *status,
                           cudaStream_t stream, bool *unsupported) {
     *unsupported = false;
+    if (decode_mma_supported(d)) {
+        cudaError_t e = launch_decode_mma(d, layer_begin, layer_count, q, k_new, v_new, new_pos, k_cache, v_cache,
+                                          score, pos, len, gamma, sm_scale, max_len, out, status, stream,
+                                          unsupported);
+        if (!*unsupported) return e;
+        *unsupported = false;  // shape outside the tensor-core kernel's limits: the generic kernel runs
+    }
     const int G = d.q_heads / d.kv_heads;
     const int units = layer_count * d.batch * d.kv_heads;
     const int nmax = (max_len > 0 && max_len < d.capacity) ? max_len : d.capacity;

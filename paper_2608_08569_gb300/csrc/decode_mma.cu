@@ -1,0 +1,522 @@
+// Fast decode step for bf16 caches (head_dim 64 or 128, GQA group <= 16): append (Eq. 1), GQA
+// attention (Eq. 2) and the decayed-score update (Eq. 6), reading each cached K and V row once.
+//
+// Grid: one thread-block cluster of S CTAs per (layer, sequence, kv-head) unit; CTA r owns the
+// token range [r*ceil(n/S), (r+1)*ceil(n/S)). Per CTA, one producer warp streams the range's K
+// tiles and then its V tiles (64 tokens each) with 2-D tensor-map TMA loads (128-byte swizzle)
+// into a 4-stage shared-memory ring guarded by mbarriers; four consumer warps take 16 tokens of
+// every tile:
+//   phase K  S = K_tile Q^T on the tensor cores (mma.sync m16n8k16, tokens as M, the group's
+//            query heads as N), scaled logits kept in shared memory, per-head CTA maximum;
+//   phase V  p = 2^(logit - max_cta), kept for the score update; O^T += V_tile^T P^T on the
+//            tensor cores with bf16 probabilities and fp32 accumulators; per-head sums.
+// One cluster exchange through distributed shared memory then gives the global per-head maximum
+// and normaliser: every CTA rewrites its tokens' scores as gamma * s + sum_h p_h / Z_h and
+// combines one slice of the G x D outputs from all CTAs' partials.
+#include <cooperative_groups.h>
+#include <cudaTypedefs.h>
+
+#include "common.cuh"
+#include "ptx.cuh"
+
+namespace cg = cooperative_groups;
+
+namespace voxzip {
+namespace {
+
+constexpr int kConsumerWarps = 4;
+constexpr int kThreads = (kConsumerWarps + 1) * 32;
+constexpr int kTile = 16 * kConsumerWarps;      // tokens per pipeline stage
+constexpr int kStages = 4;
+constexpr int kBoxCols = 64;                    // bf16 elements per TMA box row (128 bytes)
+constexpr int kBoxBytes = kTile * kBoxCols * 2;
+constexpr uint32_t kWaitLimit = 1u << 24;
+constexpr size_t kMaxSmem = 227 * 1024;
+constexpr int kMaxCluster = 16;
+
+struct MmaParams {
+    const __nv_bfloat16 *q, *k_new, *v_new;
+    const int32_t *new_pos;
+    __nv_bfloat16 *k_cache, *v_cache;
+    float *score;
+    int32_t *pos, *len;
+    __nv_bfloat16 *out;
+    int32_t *status;
+    int32_t B, L, Hq, Hkv, G, C, layer_begin, chunk_cap;
+    float gamma, scale_log2;
+};
+
+template <int D, int NT>
+struct Layout {
+    static constexpr int kHalves = D / 64;
+    static constexpr int kGP = 8 * NT;                         // heads padded to the MMA's N
+    static constexpr int kStageBytes = kHalves * kBoxBytes;
+    static constexpr int kStagesOff = 0;
+    static constexpr int kBarOff = kStages * kStageBytes;      // full[kStages], empty[kStages]
+    static constexpr int kPbufOff = kBarOff + 2 * kStages * 8;
+    static constexpr int kPbufBytes = kConsumerWarps * 16 * kGP * 2;
+    static constexpr int kOOff = kPbufOff + kPbufBytes;        // o_cta [kGP][D] fp32
+    static constexpr int kStatOff = kOOff + kGP * D * 4;       // m_w[warps][kGP], m_cta, z_cta, fac
+    static constexpr int kStatFloats = (kConsumerWarps + 3) * kGP + kMaxCluster * kGP;
+    static constexpr int kLgOff = kStatOff + kStatFloats * 4;  // logits / p [chunk_cap][kGP] fp32
+    static size_t bytes(int chunk_cap) { return 1024 + (size_t)kLgOff + (size_t)chunk_cap * kGP * 4; }
+};
+
+__device__ __forceinline__ uint32_t swz(int row, int chunk) {  // byte offset in a 128B-swizzled box
+    return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
+}
+
+template <int D, int NT>
+__global__ void __launch_bounds__(kThreads)
+decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
+                  const MmaParams p) {
+    using Lay = Layout<D, NT>;
+    constexpr int GP = Lay::kGP;
+    constexpr int kHalves = Lay::kHalves;
+    constexpr int kKSteps = D / 16;
+
+    cg::cluster_group cluster = cg::this_cluster();
+    const int S = (int)cluster.num_blocks();
+    const int rank = (int)cluster.block_rank();
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int g = lane >> 2, qd = lane & 3;
+
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t *stages = smem + Lay::kStagesOff;
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + Lay::kBarOff);
+    uint64_t *empty = full + kStages;
+    uint8_t *pbuf = smem + Lay::kPbufOff + warp * 16 * GP * 2;
+    float *o_cta = reinterpret_cast<float *>(smem + Lay::kOOff);
+    float *m_w = reinterpret_cast<float *>(smem + Lay::kStatOff);
+    float *m_cta = m_w + kConsumerWarps * GP;
+    float *z_cta = m_cta + GP;
+    float *fac_self = z_cta + GP;
+    float *fac_all = fac_self + GP;                            // [kMaxCluster][GP]
+    float *lg = reinterpret_cast<float *>(smem + Lay::kLgOff);
+
+    const UnitIdx ui = unit_of(blockIdx.y, p.B, p.L, p.Hkv, p.layer_begin);
+    const int32_t n_old = p.len[ui.cache_unit];
+    const int32_t n = n_old + 1;
+    if (n_old < 0 || n > p.C) {  // the same decision in every CTA of the cluster
+        if (rank == 0 && tid == 0) raise_status(p.status, VOXZIP_DEV_CAPACITY);
+        return;
+    }
+    const int chunk = (n + S - 1) / S;
+    if (chunk > p.chunk_cap) {
+        if (rank == 0 && tid == 0) raise_status(p.status, VOXZIP_DEV_LEN_HINT);
+        return;
+    }
+    const int j0 = min(n, rank * chunk);
+    const int cnt = min(n, j0 + chunk) - j0;
+    const int ntiles = (cnt + kTile - 1) / kTile;
+    const int64_t act_row = (int64_t)ui.l_local * p.B + ui.b;
+    const int64_t row_base = ui.cache_unit * p.C;
+
+    // Eq. 1: the CTA owning slot n-1 writes the new row; the fence orders these generic-proxy
+    // writes before the async-proxy (TMA) reads issued after the barrier below.
+    if (j0 <= n - 1 && n - 1 < j0 + cnt && tid < D / 4) {
+        const int64_t src = (act_row * p.Hkv + ui.h) * D + tid * 4;
+        const int64_t dst = (row_base + n - 1) * D + tid * 4;
+        *reinterpret_cast<uint2 *>(p.k_cache + dst) = *reinterpret_cast<const uint2 *>(p.k_new + src);
+        *reinterpret_cast<uint2 *>(p.v_cache + dst) = *reinterpret_cast<const uint2 *>(p.v_new + src);
+        if (tid == 0) p.pos[row_base + n - 1] = p.new_pos[ui.b];
+        asm volatile("fence.proxy.async.global;" ::: "memory");
+    }
+    if (tid == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            ptx::mbar_init(&full[s], 1);
+            ptx::mbar_init(&empty[s], kConsumerWarps);
+        }
+        ptx::fence_mbar_init();
+    }
+    for (int i = tid; i < GP * D; i += kThreads) o_cta[i] = 0.f;
+    for (int i = tid; i < GP; i += kThreads) z_cta[i] = 0.f;
+    __syncthreads();
+
+    bool ok = true;
+    if (warp == kConsumerWarps) {
+        // ------------------------------------------------------------- producer
+        if (lane == 0 && ntiles > 0) {
+            ptx::prefetch_tmap(&tmk);
+            ptx::prefetch_tmap(&tmv);
+            for (int i = 0; i < 2 * ntiles; ++i) {
+                const int s = i % kStages, use = i / kStages;
+                if (use > 0 && !ptx::mbar_wait_bounded(&empty[s], (use - 1) & 1, kWaitLimit)) {
+                    ok = false;
+                    break;
+                }
+                ptx::mbar_arrive_expect_tx(&full[s], Lay::kStageBytes);
+                const bool is_k = i < ntiles;
+                const int tile = is_k ? i : i - ntiles;
+                const int32_t y = (int32_t)(row_base + j0 + tile * kTile);
+                uint8_t *dst = stages + s * Lay::kStageBytes;
+#pragma unroll
+                for (int h = 0; h < kHalves; ++h)
+                    ptx::tma_load_2d(dst + h * kBoxBytes, is_k ? &tmk : &tmv, h * kBoxCols, y, &full[s]);
+            }
+        }
+        __syncwarp();  // reconverge the producer warp before the block-wide barrier
+    } else {
+        // ------------------------------------------------------------- consumers
+        // Q^T as the B operand: b0b1 = Q[head][16ks + 2qd .. +1], b2b3 = Q[head][16ks + 8 + 2qd .. +1].
+        uint32_t qb[NT][kKSteps][2];
+        const __nv_bfloat16 *qg = p.q + (act_row * p.Hq + (int64_t)ui.h * p.G) * D;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            const int head = nt * 8 + g;
+#pragma unroll
+            for (int ks = 0; ks < kKSteps; ++ks) {
+                if (head < p.G) {
+                    qb[nt][ks][0] = *reinterpret_cast<const uint32_t *>(qg + head * D + ks * 16 + 2 * qd);
+                    qb[nt][ks][1] = *reinterpret_cast<const uint32_t *>(qg + head * D + ks * 16 + 8 + 2 * qd);
+                } else {
+                    qb[nt][ks][0] = 0u;
+                    qb[nt][ks][1] = 0u;
+                }
+            }
+        }
+        float mx[NT][2];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) mx[nt][0] = mx[nt][1] = -INFINITY;
+        const int r0 = warp * 16;
+
+        // Phase K: logits of this warp's 16 tokens of every tile.
+        for (int t = 0; t < ntiles && ok; ++t) {
+            const int s = t % kStages;
+            if (!__all_sync(0xffffffffu, ptx::mbar_wait_bounded(&full[s], (t / kStages) & 1, kWaitLimit))) {
+                ok = false;
+                break;
+            }
+            const int lt0 = t * kTile + r0;
+            if (lt0 < cnt) {
+                const uint32_t base = ptx::smem_u32(stages + s * Lay::kStageBytes);
+                float acc[NT][4];
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+                const int arow = r0 + (lane & 7) + ((lane >> 3) & 1) * 8;
+#pragma unroll
+                for (int h = 0; h < kHalves; ++h) {
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        uint32_t a0, a1, a2, a3;
+                        ptx::ldsm_x4(base + h * kBoxBytes + swz(arow, kk * 2 + (lane >> 4)), a0, a1, a2, a3);
+#pragma unroll
+                        for (int nt = 0; nt < NT; ++nt)
+                            ptx::mma_bf16_16816(acc[nt], a0, a1, a2, a3, qb[nt][h * 4 + kk][0], qb[nt][h * 4 + kk][1]);
+                    }
+                }
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    const int lt = lt0 + g + half * 8;
+                    const bool valid = lt < cnt;
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt) {
+                        const float l0 = valid ? acc[nt][half * 2] * p.scale_log2 : -INFINITY;
+                        const float l1 = valid ? acc[nt][half * 2 + 1] * p.scale_log2 : -INFINITY;
+                        mx[nt][0] = fmaxf(mx[nt][0], l0);
+                        mx[nt][1] = fmaxf(mx[nt][1], l1);
+                        if (valid) *reinterpret_cast<float2 *>(lg + lt * GP + nt * 8 + 2 * qd) = make_float2(l0, l1);
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&empty[s]);
+        }
+        // CTA maximum per head.
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+                float v = mx[nt][j];
+                v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
+                v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
+                v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
+                if (g == 0) m_w[warp * GP + nt * 8 + 2 * qd + j] = v;
+            }
+        asm volatile("bar.sync 1, %0;" ::"r"(kConsumerWarps * 32) : "memory");
+        if (tid < GP) {
+            float v = -INFINITY;
+            for (int w = 0; w < kConsumerWarps; ++w) v = fmaxf(v, m_w[w * GP + tid]);
+            m_cta[tid] = v;
+        }
+        asm volatile("bar.sync 1, %0;" ::"r"(kConsumerWarps * 32) : "memory");
+
+        // Phase V: probabilities with the CTA maximum, P V on the tensor cores.
+        float oacc[kKSteps][NT][4];
+#pragma unroll
+        for (int i = 0; i < kKSteps; ++i)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) oacc[i][nt][0] = oacc[i][nt][1] = oacc[i][nt][2] = oacc[i][nt][3] = 0.f;
+        float zs[NT][2];
+        float mc[NT][2];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            zs[nt][0] = zs[nt][1] = 0.f;
+            mc[nt][0] = m_cta[nt * 8 + 2 * qd];
+            mc[nt][1] = m_cta[nt * 8 + 2 * qd + 1];
+        }
+        for (int t = 0; t < ntiles && ok; ++t) {
+            const int i = ntiles + t, s = i % kStages;
+            if (!__all_sync(0xffffffffu, ptx::mbar_wait_bounded(&full[s], (i / kStages) & 1, kWaitLimit))) {
+                ok = false;
+                break;
+            }
+            const int lt0 = t * kTile + r0;
+            if (lt0 < cnt) {
+                uint8_t *stage = stages + s * Lay::kStageBytes;
+#pragma unroll
+                for (int half = 0; half < 2; ++half) {
+                    const int lt = lt0 + g + half * 8;
+                    const bool valid = lt < cnt;
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt) {
+                        float p0 = 0.f, p1 = 0.f;
+                        if (valid) {
+                            float2 l = *reinterpret_cast<float2 *>(lg + lt * GP + nt * 8 + 2 * qd);
+                            p0 = exp2f(l.x - mc[nt][0]);
+                            p1 = exp2f(l.y - mc[nt][1]);
+                            *reinterpret_cast<float2 *>(lg + lt * GP + nt * 8 + 2 * qd) = make_float2(p0, p1);
+                        }
+                        zs[nt][0] += p0;
+                        zs[nt][1] += p1;
+                        *reinterpret_cast<uint32_t *>(pbuf + (g + half * 8) * GP * 2 + (nt * 8 + 2 * qd) * 2) =
+                            ptx::pack_bf16(p0, p1);
+                    }
+                }
+                // Rows past the range may hold anything; zero them so 0 * garbage cannot be NaN.
+                if (lt0 + 16 > cnt) {
+                    for (int e = lane; e < 16 * kHalves * 8; e += 32) {
+                        const int row = e / (kHalves * 8), rest = e % (kHalves * 8);
+                        if (lt0 + row >= cnt)
+                            *reinterpret_cast<uint4 *>(stage + (rest >> 3) * kBoxBytes + swz(r0 + row, rest & 7)) =
+                                make_uint4(0u, 0u, 0u, 0u);
+                    }
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                }
+                __syncwarp();
+                uint32_t pb[NT][2];
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt)
+                    ptx::ldsm_x2_t(ptx::smem_u32(pbuf + (lane & 15) * GP * 2 + nt * 16), pb[nt][0], pb[nt][1]);
+                const uint32_t base = ptx::smem_u32(stage);
+                const int mi = lane >> 3;
+                const int vrow = r0 + (lane & 7) + (mi >> 1) * 8;
+#pragma unroll
+                for (int h = 0; h < kHalves; ++h) {
+#pragma unroll
+                    for (int mt = 0; mt < 4; ++mt) {
+                        uint32_t a0, a1, a2, a3;
+                        ptx::ldsm_x4_t(base + h * kBoxBytes + swz(vrow, mt * 2 + (mi & 1)), a0, a1, a2, a3);
+#pragma unroll
+                        for (int nt = 0; nt < NT; ++nt)
+                            ptx::mma_bf16_16816(oacc[h * 4 + mt][nt], a0, a1, a2, a3, pb[nt][0], pb[nt][1]);
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0) ptx::mbar_arrive(&empty[s]);
+        }
+        // Per-head sums and partial outputs of this CTA.
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+                float v = zs[nt][j];
+                v += __shfl_xor_sync(0xffffffffu, v, 4);
+                v += __shfl_xor_sync(0xffffffffu, v, 8);
+                v += __shfl_xor_sync(0xffffffffu, v, 16);
+                if (g == 0) atomicAdd(&z_cta[nt * 8 + 2 * qd + j], v);
+            }
+#pragma unroll
+        for (int i = 0; i < kKSteps; ++i)
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) {
+                const int d0 = i * 16 + g, h0 = nt * 8 + 2 * qd;
+                atomicAdd(&o_cta[h0 * D + d0], oacc[i][nt][0]);
+                atomicAdd(&o_cta[(h0 + 1) * D + d0], oacc[i][nt][1]);
+                atomicAdd(&o_cta[h0 * D + d0 + 8], oacc[i][nt][2]);
+                atomicAdd(&o_cta[(h0 + 1) * D + d0 + 8], oacc[i][nt][3]);
+            }
+    }
+    if (!ok) raise_status(p.status, VOXZIP_DEV_TIMEOUT);
+    __syncthreads();
+    cluster.sync();  // every CTA's m_cta, z_cta, o_cta are final
+
+    // Global per-head maximum and normaliser; fac_all[r][h] = 2^(m_r - m) / Z.
+    if (tid < GP) {
+        float m = -INFINITY;
+        for (int r = 0; r < S; ++r) m = fmaxf(m, *cluster.map_shared_rank(&m_cta[tid], r));
+        float z = 0.f;
+        for (int r = 0; r < S; ++r) {
+            const float mr = *cluster.map_shared_rank(&m_cta[tid], r);
+            const float e = mr == -INFINITY ? 0.f : exp2f(mr - m);
+            fac_all[r * GP + tid] = e;
+            z += e * *cluster.map_shared_rank(&z_cta[tid], r);
+        }
+        const float rz = 1.f / z;
+        for (int r = 0; r < S; ++r) fac_all[r * GP + tid] *= rz;
+        fac_self[tid] = fac_all[rank * GP + tid];
+    }
+    __syncthreads();
+
+    // Eq. 6 for this CTA's tokens: A = gamma * [A, 0] + sum over the group's heads.
+    {
+        float *sc = p.score + row_base;
+        for (int i = tid; i < cnt; i += kThreads) {
+            const int j = j0 + i;
+            const float prev = (j == n - 1) ? 0.f : sc[j];
+            float add = 0.f;
+            const float *pr = lg + i * GP;
+#pragma unroll
+            for (int h = 0; h < GP; ++h)
+                if (h < p.G) add += pr[h] * fac_self[h];
+            sc[j] = p.gamma * prev + add;
+        }
+    }
+    // Combine the partial outputs; CTA r writes slice r of the G x D outputs.
+    {
+        const int total = p.G * D, per = (total + S - 1) / S;
+        const int lo = rank * per, hi = min(total, lo + per);
+        __nv_bfloat16 *og = p.out + (act_row * p.Hq + (int64_t)ui.h * p.G) * D;
+        for (int i = lo + tid; i < hi; i += kThreads) {
+            const int h = i / D;
+            float o = 0.f;
+            for (int r = 0; r < S; ++r) o += fac_all[r * GP + h] * *cluster.map_shared_rank(&o_cta[i], r);
+            og[i] = __float2bfloat16_rn(o);
+        }
+    }
+    cluster.sync();  // no CTA leaves while others may still read its shared memory
+    if (rank == 0 && tid == 0) p.len[ui.cache_unit] = n;
+}
+
+// ---------------------------------------------------------------- host side
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (fn == nullptr) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+    }
+    return fn;
+}
+
+// The whole cache as a 2-D [rows][D] bf16 tensor; boxes of kTile rows x 64 columns, 128B swizzle.
+bool make_map(CUtensorMap *map, void *base, int64_t rows, int D) {
+    auto enc = tensor_map_encoder();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)D * 2};
+    cuuint32_t box[2] = {(cuuint32_t)kBoxCols, (cuuint32_t)kTile};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int D, int NT>
+cudaError_t launch_t(const CUtensorMap &tmk, const CUtensorMap &tmv, const MmaParams &prm, int S, int units,
+                     cudaStream_t stream) {
+    auto kern = decode_mma_kernel<D, NT>;
+    static bool configured = false;
+    if (!configured) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem);
+        if (e != cudaSuccess) return e;
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+        configured = true;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)S, (unsigned)units, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = Layout<D, NT>::bytes(prm.chunk_cap);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, tmk, tmv, prm);
+}
+
+}  // namespace
+
+// Returns false when this path does not apply (fp32 cache, other head dims, group > 16).
+bool decode_mma_supported(const voxzip_cache_desc &d) {
+    const int G = d.q_heads / d.kv_heads;
+    return d.dtype == VOXZIP_BF16 && (d.head_dim == 64 || d.head_dim == 128) && G >= 1 && G <= 16 &&
+           tensor_map_encoder() != nullptr;
+}
+
+cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, int32_t layer_count, const void *q,
+                              const void *k_new, const void *v_new, const int32_t *new_pos, void *k_cache,
+                              void *v_cache, float *score, int32_t *pos, int32_t *len, float gamma, float sm_scale,
+                              int32_t max_len, void *out, int32_t *status, cudaStream_t stream, bool *unsupported) {
+    *unsupported = false;
+    const int G = d.q_heads / d.kv_heads;
+    const int NT = G <= 8 ? 1 : 2;
+    const int units = layer_count * d.batch * d.kv_heads;
+    const int nmax = (max_len > 0 && max_len < d.capacity) ? max_len : d.capacity;
+    // Split so that the grid has at least ~4 CTAs per SM of work and no CTA exceeds ~1024 tokens.
+    int sms = 148;
+    {
+        int dev = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    }
+    int S = 1;
+    while (S < kMaxCluster && ((int64_t)units * S < 4LL * sms || (nmax + S - 1) / S > 1024) &&
+           (nmax + 2 * S - 1) / (2 * S) >= kTile)
+        S <<= 1;
+    while (S < kMaxCluster && (nmax + S - 1) / S > 1024) S <<= 1;
+    const int chunk_cap = (nmax + S - 1) / S;
+    const size_t smem = d.head_dim == 128 ? (NT == 1 ? Layout<128, 1>::bytes(chunk_cap) : Layout<128, 2>::bytes(chunk_cap))
+                                          : (NT == 1 ? Layout<64, 1>::bytes(chunk_cap) : Layout<64, 2>::bytes(chunk_cap));
+    if (smem > kMaxSmem) {
+        *unsupported = true;
+        return cudaSuccess;
+    }
+    const int64_t rows = (int64_t)d.batch * d.layers * d.kv_heads * d.capacity;
+    thread_local void *cached_k = nullptr, *cached_v = nullptr;
+    thread_local int64_t cached_rows = 0;
+    thread_local int cached_d = 0;
+    thread_local CUtensorMap tmk, tmv;
+    if (cached_k != k_cache || cached_v != v_cache || cached_rows != rows || cached_d != d.head_dim) {
+        if (!make_map(&tmk, k_cache, rows, d.head_dim) || !make_map(&tmv, v_cache, rows, d.head_dim)) {
+            cached_k = cached_v = nullptr;
+            *unsupported = true;
+            return cudaSuccess;
+        }
+        cached_k = k_cache;
+        cached_v = v_cache;
+        cached_rows = rows;
+        cached_d = d.head_dim;
+    }
+    MmaParams prm;
+    prm.q = static_cast<const __nv_bfloat16 *>(q);
+    prm.k_new = static_cast<const __nv_bfloat16 *>(k_new);
+    prm.v_new = static_cast<const __nv_bfloat16 *>(v_new);
+    prm.new_pos = new_pos;
+    prm.k_cache = static_cast<__nv_bfloat16 *>(k_cache);
+    prm.v_cache = static_cast<__nv_bfloat16 *>(v_cache);
+    prm.score = score;
+    prm.pos = pos;
+    prm.len = len;
+    prm.out = static_cast<__nv_bfloat16 *>(out);
+    prm.status = status;
+    prm.B = d.batch; prm.L = d.layers; prm.Hq = d.q_heads; prm.Hkv = d.kv_heads; prm.G = G;
+    prm.C = d.capacity; prm.layer_begin = layer_begin; prm.chunk_cap = chunk_cap;
+    prm.gamma = gamma;
+    const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)d.head_dim);
+    prm.scale_log2 = scale * 1.4426950408889634f;  // log2(e): exp(x) = 2^(x log2 e)
+    if (d.head_dim == 128)
+        return NT == 1 ? launch_t<128, 1>(tmk, tmv, prm, S, units, stream)
+                       : launch_t<128, 2>(tmk, tmv, prm, S, units, stream);
+    return NT == 1 ? launch_t<64, 1>(tmk, tmv, prm, S, units, stream) : launch_t<64, 2>(tmk, tmv, prm, S, units, stream);
+}
+
+}  // namespace voxzip

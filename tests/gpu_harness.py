@@ -175,6 +175,7 @@ def check_units(w, rec, orc_results, sample, steps=None):
     tol = out_tol(w)
     assert rec["status"] == 0, f"device status bits {rec['status']:#x}"
     diverged = []
+    stats = dict(max_out_err=0.0, max_score_rel=0.0, evictions=0)
     for i, ((b, l, h), o) in enumerate(zip(sample, orc_results)):
         bud = w.budget[b]
         M = math.floor(float(np.float32(w.recent_frac)) * bud)
@@ -183,6 +184,7 @@ def check_units(w, rec, orc_results, sample, steps=None):
         gone = False
         for t in range(1, S + 1):
             err = np.abs(rec["out"][t - 1, i] - o["out"][t - 1]).max()
+            stats["max_out_err"] = max(stats["max_out_err"], float(err))
             assert err <= tol, f"unit {(b, l, h)} step {t}: output error {err:.3g} > {tol}"
             if t % w.interval:
                 continue
@@ -190,6 +192,9 @@ def check_units(w, rec, orc_results, sample, steps=None):
             assert rec["len_before"][ev, i] == n, f"unit {(b, l, h)} eviction {ev}: length"
             gs, os_ = rec["score_before"][ev, i, :n], o["score_before"][ev, :n]
             bad = np.abs(gs - os_) > SCORE_RTOL * np.abs(os_) + SCORE_ATOL
+            stats["max_score_rel"] = max(stats["max_score_rel"], float(
+                (np.abs(gs - os_) / np.maximum(np.abs(os_), 1e-30)).max()))
+            stats["evictions"] += 1
             assert not bad.any(), (f"unit {(b, l, h)} eviction {ev}: {bad.sum()} scores off, worst rel "
                                    f"{(np.abs(gs - os_) / np.maximum(np.abs(os_), 1e-30)).max():.3g}")
             m = min(n, bud)
@@ -210,4 +215,5 @@ def check_units(w, rec, orc_results, sample, steps=None):
         np.testing.assert_allclose(rec["score"][i, :n], o["score"], rtol=SCORE_RTOL, atol=SCORE_ATOL)
         np.testing.assert_array_equal(rec["k"][i, :n].double().numpy(), o["K"])
         np.testing.assert_array_equal(rec["v"][i, :n].double().numpy(), o["V"])
+    check_units.last_stats = stats
     return diverged

@@ -39,6 +39,10 @@ def _pipeline(w, sample_k, steps=None, anchors=False):
     check_stage1(w, inp, rec, sample, anchors=anc)
     res = oracle_units(w, inp, sample, steps=steps, anchors=anc)
     diverged = check_units(w, rec, res, sample, steps=steps)
+    st = check_units.last_stats
+    print(f"\n[parity] {w.name}: {len(sample)} units, {st['evictions']} evictions compared, "
+          f"max |out err| {st['max_out_err']:.3g}, max score rel err {st['max_score_rel']:.3g}, "
+          f"diverged at near-ties: {diverged}")
     assert len(diverged) <= max(1, len(sample) // 4), diverged
     return rec, res, diverged
 
