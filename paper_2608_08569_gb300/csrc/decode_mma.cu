@@ -24,10 +24,20 @@ namespace cg = cooperative_groups;
 namespace voxzip {
 namespace {
 
-constexpr int kConsumerWarps = 4;
+#ifndef VOXZIP_DECODE_WARPS
+#define VOXZIP_DECODE_WARPS 4      // consumer warps per CTA (16 tokens of every tile each)
+#endif
+#ifndef VOXZIP_DECODE_STAGES
+#define VOXZIP_DECODE_STAGES 3     // depth of the shared-memory tile ring
+#endif
+#ifndef VOXZIP_DECODE_CTA_OVERHEAD
+#define VOXZIP_DECODE_CTA_OVERHEAD 384  // fixed cost of one CTA in the split model, in tokens streamed
+#endif
+
+constexpr int kConsumerWarps = VOXZIP_DECODE_WARPS;
 constexpr int kThreads = (kConsumerWarps + 1) * 32;
 constexpr int kTile = 16 * kConsumerWarps;      // tokens per pipeline stage
-constexpr int kStages = 4;
+constexpr int kStages = VOXZIP_DECODE_STAGES;
 constexpr int kBoxCols = 64;                    // bf16 elements per TMA box row (128 bytes)
 constexpr int kBoxBytes = kTile * kBoxCols * 2;
 constexpr uint32_t kWaitLimit = 1u << 24;
@@ -51,15 +61,18 @@ struct Layout {
     static constexpr int kHalves = D / 64;
     static constexpr int kGP = 8 * NT;                         // heads padded to the MMA's N
     static constexpr int kStageBytes = kHalves * kBoxBytes;
-    static constexpr int kStagesOff = 0;
-    static constexpr int kBarOff = kStages * kStageBytes;      // full[kStages], empty[kStages]
+    static constexpr int kStagesOff = 0;                       // the ring; reused for o_w afterwards
+    static constexpr int kRingBytes = kStages * kStageBytes;
+    static_assert(kRingBytes >= kConsumerWarps * kGP * D * 4, "ring too small to hold the warp partials");
+    static constexpr int kBarOff = kRingBytes;                 // full[kStages], empty[kStages]
     static constexpr int kPbufOff = kBarOff + 2 * kStages * 8;
     static constexpr int kPbufBytes = kConsumerWarps * 16 * kGP * 2;
-    static constexpr int kOOff = kPbufOff + kPbufBytes;        // o_cta [kGP][D] fp32
-    static constexpr int kStatOff = kOOff + kGP * D * 4;       // m_w[warps][kGP], m_cta, z_cta, fac
-    static constexpr int kStatFloats = (kConsumerWarps + 3) * kGP + kMaxCluster * kGP;
-    static constexpr int kLgOff = kStatOff + kStatFloats * 4;  // logits / p [chunk_cap][kGP] fp32
-    static size_t bytes(int chunk_cap) { return 1024 + (size_t)kLgOff + (size_t)chunk_cap * kGP * 4; }
+    static constexpr int kStatOff = kPbufOff + kPbufBytes;     // m_w[warps][kGP], z_w[warps][kGP], m_cta, z_cta, fac
+    static constexpr int kStatFloats = (2 * kConsumerWarps + 3) * kGP + kMaxCluster * kGP;
+    static constexpr int kLgOff = kStatOff + kStatFloats * 4;  // logits / p [chunk_cap][kGP] fp32, then old scores
+    static size_t bytes(int chunk_cap) {
+        return 1024 + (size_t)kLgOff + (size_t)chunk_cap * kGP * 4 + (size_t)chunk_cap * 4;
+    }
 };
 
 __device__ __forceinline__ uint32_t swz(int row, int chunk) {  // byte offset in a 128B-swizzled box
@@ -87,13 +100,16 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + Lay::kBarOff);
     uint64_t *empty = full + kStages;
     uint8_t *pbuf = smem + Lay::kPbufOff + warp * 16 * GP * 2;
-    float *o_cta = reinterpret_cast<float *>(smem + Lay::kOOff);
+    float *o_w = reinterpret_cast<float *>(stages);            // [warps][GP][D], valid after the ring drains
+    float *o_cta = o_w;                                        // the sum over warps lands in warp 0's slot
     float *m_w = reinterpret_cast<float *>(smem + Lay::kStatOff);
-    float *m_cta = m_w + kConsumerWarps * GP;
+    float *z_w = m_w + kConsumerWarps * GP;
+    float *m_cta = z_w + kConsumerWarps * GP;
     float *z_cta = m_cta + GP;
     float *fac_self = z_cta + GP;
     float *fac_all = fac_self + GP;                            // [kMaxCluster][GP]
     float *lg = reinterpret_cast<float *>(smem + Lay::kLgOff);
+    float *s_old = lg + (size_t)p.chunk_cap * GP;               // [chunk_cap] scores before the step
 
     const UnitIdx ui = unit_of(blockIdx.y, p.B, p.L, p.Hkv, p.layer_begin);
     const int32_t n_old = p.len[ui.cache_unit];
@@ -130,8 +146,14 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         }
         ptx::fence_mbar_init();
     }
-    for (int i = tid; i < GP * D; i += kThreads) o_cta[i] = 0.f;
-    for (int i = tid; i < GP; i += kThreads) z_cta[i] = 0.f;
+    // The old scores of this CTA's tokens travel to shared memory while the tiles stream.
+    if (warp < kConsumerWarps) {
+        const float *src = p.score + row_base + j0;
+        for (int i = tid; i < cnt; i += kConsumerWarps * 32)
+            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(ptx::smem_u32(s_old + i)), "l"(src + i)
+                         : "memory");
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    }
     __syncthreads();
 
     bool ok = true;
@@ -317,7 +339,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&empty[s]);
         }
-        // Per-head sums and partial outputs of this CTA.
+        // Per-head sums and partial outputs of this warp, then of the CTA (fixed summation order).
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
@@ -326,18 +348,34 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                 v += __shfl_xor_sync(0xffffffffu, v, 4);
                 v += __shfl_xor_sync(0xffffffffu, v, 8);
                 v += __shfl_xor_sync(0xffffffffu, v, 16);
-                if (g == 0) atomicAdd(&z_cta[nt * 8 + 2 * qd + j], v);
+                if (g == 0) z_w[warp * GP + nt * 8 + 2 * qd + j] = v;
             }
+        asm volatile("bar.sync 1, %0;" ::"r"(kConsumerWarps * 32) : "memory");  // the ring is drained
+        float *ow = o_w + warp * GP * D;
 #pragma unroll
         for (int i = 0; i < kKSteps; ++i)
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
                 const int d0 = i * 16 + g, h0 = nt * 8 + 2 * qd;
-                atomicAdd(&o_cta[h0 * D + d0], oacc[i][nt][0]);
-                atomicAdd(&o_cta[(h0 + 1) * D + d0], oacc[i][nt][1]);
-                atomicAdd(&o_cta[h0 * D + d0 + 8], oacc[i][nt][2]);
-                atomicAdd(&o_cta[(h0 + 1) * D + d0 + 8], oacc[i][nt][3]);
+                ow[h0 * D + d0] = oacc[i][nt][0];
+                ow[(h0 + 1) * D + d0] = oacc[i][nt][1];
+                ow[h0 * D + d0 + 8] = oacc[i][nt][2];
+                ow[(h0 + 1) * D + d0 + 8] = oacc[i][nt][3];
             }
+        asm volatile("bar.sync 1, %0;" ::"r"(kConsumerWarps * 32) : "memory");
+        for (int e = tid; e < GP * D; e += kConsumerWarps * 32) {
+            float v = o_w[e];
+#pragma unroll
+            for (int w = 1; w < kConsumerWarps; ++w) v += o_w[w * GP * D + e];
+            o_cta[e] = v;
+        }
+        if (tid < GP) {
+            float v = 0.f;
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) v += z_w[w * GP + tid];
+            z_cta[tid] = v;
+        }
+        asm volatile("cp.async.wait_all;" ::: "memory");
     }
     if (!ok) raise_status(p.status, VOXZIP_DEV_TIMEOUT);
     __syncthreads();
@@ -345,17 +383,25 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
 
     // Global per-head maximum and normaliser; fac_all[r][h] = 2^(m_r - m) / Z.
     if (tid < GP) {
+        float mr[kMaxCluster], zr[kMaxCluster];
+#pragma unroll
+        for (int r = 0; r < kMaxCluster; ++r) {
+            mr[r] = r < S ? *cluster.map_shared_rank(&m_cta[tid], r) : -INFINITY;
+            zr[r] = r < S ? *cluster.map_shared_rank(&z_cta[tid], r) : 0.f;
+        }
         float m = -INFINITY;
-        for (int r = 0; r < S; ++r) m = fmaxf(m, *cluster.map_shared_rank(&m_cta[tid], r));
+#pragma unroll
+        for (int r = 0; r < kMaxCluster; ++r) m = fmaxf(m, mr[r]);
         float z = 0.f;
-        for (int r = 0; r < S; ++r) {
-            const float mr = *cluster.map_shared_rank(&m_cta[tid], r);
-            const float e = mr == -INFINITY ? 0.f : exp2f(mr - m);
-            fac_all[r * GP + tid] = e;
-            z += e * *cluster.map_shared_rank(&z_cta[tid], r);
+#pragma unroll
+        for (int r = 0; r < kMaxCluster; ++r) {
+            mr[r] = mr[r] == -INFINITY ? 0.f : exp2f(mr[r] - m);
+            z += mr[r] * zr[r];
         }
         const float rz = 1.f / z;
-        for (int r = 0; r < S; ++r) fac_all[r * GP + tid] *= rz;
+#pragma unroll
+        for (int r = 0; r < kMaxCluster; ++r)
+            if (r < S) fac_all[r * GP + tid] = mr[r] * rz;
         fac_self[tid] = fac_all[rank * GP + tid];
     }
     __syncthreads();
@@ -365,7 +411,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         float *sc = p.score + row_base;
         for (int i = tid; i < cnt; i += kThreads) {
             const int j = j0 + i;
-            const float prev = (j == n - 1) ? 0.f : sc[j];
+            const float prev = (j == n - 1) ? 0.f : s_old[i];
             float add = 0.f;
             const float *pr = lg + i * GP;
 #pragma unroll
@@ -381,8 +427,13 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         __nv_bfloat16 *og = p.out + (act_row * p.Hq + (int64_t)ui.h * p.G) * D;
         for (int i = lo + tid; i < hi; i += kThreads) {
             const int h = i / D;
+            float part[kMaxCluster];
+#pragma unroll
+            for (int r = 0; r < kMaxCluster; ++r) part[r] = r < S ? *cluster.map_shared_rank(&o_cta[i], r) : 0.f;
             float o = 0.f;
-            for (int r = 0; r < S; ++r) o += fac_all[r * GP + h] * *cluster.map_shared_rank(&o_cta[i], r);
+#pragma unroll
+            for (int r = 0; r < kMaxCluster; ++r)
+                if (r < S) o += fac_all[r * GP + h] * part[r];
             og[i] = __float2bfloat16_rn(o);
         }
     }
@@ -418,17 +469,46 @@ bool make_map(CUtensorMap *map, void *base, int64_t rows, int D) {
 }
 
 template <int D, int NT>
+bool configure() {  // kernel attributes are per function; set once per process
+    static bool done = false;
+    if (!done) {
+        auto kern = decode_mma_kernel<D, NT>;
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem) != cudaSuccess ||
+            cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
+            return false;
+        done = true;
+    }
+    return true;
+}
+
+// Resident CTAs per SM for a given dynamic shared-memory size (cached: the candidates repeat).
+template <int D, int NT>
+int occupancy_t(size_t smem) {
+    thread_local size_t last_smem[8] = {};
+    thread_local int last_occ[8] = {};
+    thread_local int next = 0;
+    for (int i = 0; i < 8; ++i)
+        if (last_smem[i] == smem) return last_occ[i];
+    if (!configure<D, NT>()) return 0;
+    int occ = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, decode_mma_kernel<D, NT>, kThreads, smem) != cudaSuccess)
+        occ = 0;
+    last_smem[next] = smem;
+    last_occ[next] = occ;
+    next = (next + 1) % 8;
+    return occ;
+}
+
+int occupancy(int D, int NT, size_t smem) {
+    if (D == 128) return NT == 1 ? occupancy_t<128, 1>(smem) : occupancy_t<128, 2>(smem);
+    return NT == 1 ? occupancy_t<64, 1>(smem) : occupancy_t<64, 2>(smem);
+}
+
+template <int D, int NT>
 cudaError_t launch_t(const CUtensorMap &tmk, const CUtensorMap &tmv, const MmaParams &prm, int S, int units,
                      cudaStream_t stream) {
     auto kern = decode_mma_kernel<D, NT>;
-    static bool configured = false;
-    if (!configured) {
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem);
-        if (e != cudaSuccess) return e;
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
-        if (e != cudaSuccess) return e;
-        configured = true;
-    }
+    if (!configure<D, NT>()) return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)S, (unsigned)units, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
@@ -462,24 +542,39 @@ cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, i
     const int NT = G <= 8 ? 1 : 2;
     const int units = layer_count * d.batch * d.kv_heads;
     const int nmax = (max_len > 0 && max_len < d.capacity) ? max_len : d.capacity;
-    // Split so that the grid has at least ~4 CTAs per SM of work and no CTA exceeds ~1024 tokens.
+    // Cluster size: for each candidate S, CTAs hold ceil(nmax/S) tokens; the occupancy API gives how
+    // many fit an SM with that much shared memory, and the cost is the number of CTA waves times
+    // (tokens per CTA + a fixed per-CTA overhead), plus one CTA's worth of tail.
     int sms = 148;
     {
         int dev = 0;
         if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     }
-    int S = 1;
-    while (S < kMaxCluster && ((int64_t)units * S < 4LL * sms || (nmax + S - 1) / S > 1024) &&
-           (nmax + 2 * S - 1) / (2 * S) >= kTile)
-        S <<= 1;
-    while (S < kMaxCluster && (nmax + S - 1) / S > 1024) S <<= 1;
-    const int chunk_cap = (nmax + S - 1) / S;
-    const size_t smem = d.head_dim == 128 ? (NT == 1 ? Layout<128, 1>::bytes(chunk_cap) : Layout<128, 2>::bytes(chunk_cap))
-                                          : (NT == 1 ? Layout<64, 1>::bytes(chunk_cap) : Layout<64, 2>::bytes(chunk_cap));
-    if (smem > kMaxSmem) {
+    auto smem_of = [&](int cap) {
+        return d.head_dim == 128 ? (NT == 1 ? Layout<128, 1>::bytes(cap) : Layout<128, 2>::bytes(cap))
+                                 : (NT == 1 ? Layout<64, 1>::bytes(cap) : Layout<64, 2>::bytes(cap));
+    };
+    int S = 0;
+    double best = 0.0;
+    for (int s = 1; s <= kMaxCluster; s <<= 1) {
+        const int cap = (nmax + s - 1) / s;
+        if (s > 1 && cap < kTile / 2) break;
+        const size_t sm = smem_of(cap);
+        if (sm > kMaxSmem) continue;
+        const int occ = occupancy(d.head_dim, NT, sm);
+        if (occ <= 0) continue;
+        const double per_cta = (double)cap + VOXZIP_DECODE_CTA_OVERHEAD;
+        const double cost = (double)units * s * per_cta / ((double)sms * occ) + per_cta;
+        if (S == 0 || cost < best) {
+            S = s;
+            best = cost;
+        }
+    }
+    if (S == 0) {
         *unsupported = true;
         return cudaSuccess;
     }
+    const int chunk_cap = (nmax + S - 1) / S;
     const int64_t rows = (int64_t)d.batch * d.layers * d.kv_heads * d.capacity;
     thread_local void *cached_k = nullptr, *cached_v = nullptr;
     thread_local int64_t cached_rows = 0;
