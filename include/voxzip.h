@@ -47,7 +47,9 @@ typedef enum {
     VOXZIP_OK = 0,
     VOXZIP_EINVAL = 1,       /* invalid argument; nothing was launched */
     VOXZIP_EUNSUPPORTED = 2, /* valid request outside what the kernels implement */
-    VOXZIP_ECUDA = 3         /* a CUDA runtime call or kernel launch failed */
+    VOXZIP_ECUDA = 3,        /* a CUDA runtime call or kernel launch failed */
+    VOXZIP_ESCRATCH = 4      /* the request needs more scratch than voxzip_anchor_fuse_noalloc's
+                                fixed 4 MiB; nothing was launched */
 } voxzip_status;
 
 /* Bits of the device status word (asynchronous errors). */
@@ -112,6 +114,33 @@ voxzip_status voxzip_anchor_fuse(const voxzip_cache_desc *desc, const void *k_pr
 /* Bytes of workspace voxzip_anchor_fuse needs (0 if the descriptor is invalid). */
 size_t voxzip_anchor_fuse_workspace_size(const voxzip_cache_desc *desc, int32_t prefill_stride,
                                          int32_t num_spans);
+
+/*
+ * Stage 1 exactly as voxzip_anchor_fuse, but without a workspace argument: for callers that cannot
+ * allocate device memory, such as a runtime whose device memory belongs entirely to another
+ * framework's pool, or an audio front-end that must not allocate while it serves requests. The
+ * paper has no counterpart; this is a deployment variant of the same computation.
+ *
+ * Its scratch is a fixed 4 MiB array compiled into the library, held by every GPU that loads the
+ * library until the process exits. A request whose voxzip_anchor_fuse_workspace_size exceeds 4 MiB
+ * returns VOXZIP_ESCRATCH and launches nothing. The need is about 8 bytes per prompt token plus
+ * 8 per span, so 4 MiB covers for instance 32 sequences of 10 000 tokens or 4 of 80 000.
+ *   - The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
+ *     that device current; make that first call before any stream capture.
+ *   - Every call on a device shares the array and it keeps the last call's contents; no part of it
+ *     needs to start at zero. Calls that overlap on the GPU (unordered streams) race on it.
+ * Arguments, layouts, results and device errors are those of voxzip_anchor_fuse.
+ */
+voxzip_status voxzip_anchor_fuse_noalloc(const voxzip_cache_desc *desc, const void *k_prefill,
+                                         const void *v_prefill, int32_t prefill_stride,
+                                         const int32_t *in_len, const int32_t *audio_begin,
+                                         const int32_t *audio_len, const int32_t *span_off,
+                                         int32_t num_spans, const int32_t *span_start,
+                                         const int32_t *span_end, const int32_t *span_groups,
+                                         const void *anchor_k, const void *anchor_v,
+                                         int32_t anchor_stride, void *k_cache, void *v_cache,
+                                         float *score, int32_t *pos, int32_t *len,
+                                         int32_t *slot_map, voxzip_stream_t stream);
 
 /*
  * One decode step for layers [layer_begin, layer_begin + layer_count) of every sequence:

@@ -6,12 +6,12 @@ The three steps of the path (arxiv 2608.08569, Sec. 3.2):
   voxzip_evict         sinks + recent window + top-N history, compacted in place (Eq. 7-9)
 """
 from ._native import (CacheDesc, VoxZipError, allocate_cache, lib, voxzip_anchor_fuse,
-                      voxzip_anchor_fuse_workspace_size, voxzip_decode_step, voxzip_evict,
+                      voxzip_anchor_fuse_noalloc, voxzip_anchor_fuse_workspace_size, voxzip_decode_step, voxzip_evict,
                       voxzip_get_status)
-from ._native import (DEV_BAD_BUDGET, DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, VOXZIP_ECUDA,
-                      VOXZIP_EINVAL, VOXZIP_EUNSUPPORTED, VOXZIP_OK)
+from ._native import (DEV_BAD_BUDGET, DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_TIMEOUT, VOXZIP_ECUDA,
+                      VOXZIP_EINVAL, VOXZIP_ESCRATCH, VOXZIP_EUNSUPPORTED, VOXZIP_OK)
 
-__all__ = ["CacheDesc", "VoxZipError", "allocate_cache", "lib", "voxzip_anchor_fuse",
+__all__ = ["CacheDesc", "VoxZipError", "allocate_cache", "lib", "voxzip_anchor_fuse", "voxzip_anchor_fuse_noalloc",
            "voxzip_anchor_fuse_workspace_size", "voxzip_decode_step", "voxzip_evict", "voxzip_get_status",
-           "DEV_BAD_BUDGET", "DEV_BAD_SPANS", "DEV_CAPACITY", "DEV_LEN_HINT", "VOXZIP_ECUDA", "VOXZIP_EINVAL",
-           "VOXZIP_EUNSUPPORTED", "VOXZIP_OK"]
+           "DEV_BAD_BUDGET", "DEV_BAD_SPANS", "DEV_CAPACITY", "DEV_LEN_HINT", "DEV_TIMEOUT", "VOXZIP_ECUDA",
+           "VOXZIP_EINVAL", "VOXZIP_ESCRATCH", "VOXZIP_EUNSUPPORTED", "VOXZIP_OK"]

@@ -15,7 +15,7 @@ import torch
 
 from .build import LIB_PATH
 
-VOXZIP_OK, VOXZIP_EINVAL, VOXZIP_EUNSUPPORTED, VOXZIP_ECUDA = 0, 1, 2, 3
+VOXZIP_OK, VOXZIP_EINVAL, VOXZIP_EUNSUPPORTED, VOXZIP_ECUDA, VOXZIP_ESCRATCH = 0, 1, 2, 3, 4
 DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_BAD_BUDGET, DEV_TIMEOUT = 0x1, 0x2, 0x4, 0x8, 0x10
 VOXZIP_F32, VOXZIP_BF16 = 0, 1
 
@@ -73,6 +73,9 @@ def lib() -> ctypes.CDLL:
             L = ctypes.CDLL(LIB_PATH)
             L.voxzip_anchor_fuse.argtypes = [_DP, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _vp,
                                              _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+            L.voxzip_anchor_fuse_noalloc.argtypes = [_DP, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp,
+                                                     _vp, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp]
+            L.voxzip_anchor_fuse_noalloc.restype = _i32
             L.voxzip_anchor_fuse_workspace_size.argtypes = [_DP, _i32, _i32]
             L.voxzip_anchor_fuse_workspace_size.restype = _sz
             L.voxzip_decode_step.argtypes = [_DP, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
@@ -173,6 +176,39 @@ def voxzip_anchor_fuse(desc: CacheDesc, k_prefill, v_prefill, in_len, audio_begi
         _ptr(audio_len), _ptr(span_off), int(num_spans), _ptr(span_start), _ptr(span_end), _ptr(span_groups),
         _ptr(anchor_k), _ptr(anchor_v), int(anchor_stride), _ptr(k_cache), _ptr(v_cache), _ptr(score),
         _ptr(pos), _ptr(len_), _ptr(slot_map), _ptr(workspace), int(workspace.numel()), _stream(stream)))
+
+
+def voxzip_anchor_fuse_noalloc(desc: CacheDesc, k_prefill, v_prefill, in_len, audio_begin, audio_len, span_off,
+                               span_start, span_end, span_groups, k_cache, v_cache, score, pos, len_, *,
+                               slot_map=None, anchor_k=None, anchor_v=None, stream=None) -> None:
+    """Stage 1 like voxzip_anchor_fuse, for callers that cannot allocate: the library's fixed
+    4 MiB scratch replaces the workspace (VoxZipError with VOXZIP_ESCRATCH if it is too small)."""
+    B, L, H, D = desc.batch, desc.layers, desc.kv_heads, desc.head_dim
+    if k_prefill.dim() != 5:
+        raise ValueError("k_prefill must be [B][L][Hkv][stride][D]")
+    stride = k_prefill.shape[3]
+    _need(k_prefill, "k_prefill", desc.dtype, (B, L, H, stride, D))
+    _need(v_prefill, "v_prefill", desc.dtype, (B, L, H, stride, D))
+    for name, t in (("in_len", in_len), ("audio_begin", audio_begin), ("audio_len", audio_len)):
+        _need(t, name, torch.int32, (B,))
+    _need(span_off, "span_off", torch.int32, (B + 1,))
+    num_spans = span_start.numel()
+    for name, t in (("span_start", span_start), ("span_end", span_end), ("span_groups", span_groups)):
+        _need(t, name, torch.int32, (num_spans,))
+    _check_cache(desc, k_cache, v_cache, score, pos, len_)
+    if slot_map is not None:
+        _need(slot_map, "slot_map", torch.int32, (B, stride))
+    anchor_stride = 0
+    if anchor_k is not None or anchor_v is not None:
+        anchor_stride = anchor_k.shape[3]
+        _need(anchor_k, "anchor_k", desc.dtype, (B, L, H, anchor_stride, D))
+        _need(anchor_v, "anchor_v", desc.dtype, (B, L, H, anchor_stride, D))
+    d = desc.c_struct()
+    _check("voxzip_anchor_fuse_noalloc", lib().voxzip_anchor_fuse_noalloc(
+        ctypes.byref(d), _ptr(k_prefill), _ptr(v_prefill), int(stride), _ptr(in_len), _ptr(audio_begin),
+        _ptr(audio_len), _ptr(span_off), int(num_spans), _ptr(span_start), _ptr(span_end), _ptr(span_groups),
+        _ptr(anchor_k), _ptr(anchor_v), int(anchor_stride), _ptr(k_cache), _ptr(v_cache), _ptr(score),
+        _ptr(pos), _ptr(len_), _ptr(slot_map), _stream(stream)))
 
 
 def voxzip_decode_step(desc: CacheDesc, layer_begin: int, layer_count: int, q, k_new, v_new, new_pos,

@@ -45,6 +45,9 @@ constexpr int kMaxGridY = 65535;
 
 }  // namespace
 
+// The status word's device address on the current device, for entry points in other files.
+voxzip_status voxzip_status_word_address(int32_t **addr) { return status_word(addr); }
+
 extern "C" {
 
 int32_t voxzip_version(void) { return 100; }
@@ -55,6 +58,7 @@ const char *voxzip_status_string(voxzip_status s) {
         case VOXZIP_EINVAL: return "VOXZIP_EINVAL";
         case VOXZIP_EUNSUPPORTED: return "VOXZIP_EUNSUPPORTED";
         case VOXZIP_ECUDA: return "VOXZIP_ECUDA";
+        case VOXZIP_ESCRATCH: return "VOXZIP_ESCRATCH";
     }
     return "VOXZIP_UNKNOWN";
 }
