@@ -57,6 +57,26 @@ def cores() -> int:
         return os.cpu_count() or 1
 
 
+def profiled_traffic_ratio(profile: str, sources) -> float | None:
+    """DRAM traffic / algorithmic bytes from a committed ncu summary, or None when the kernel's
+    sources changed since that capture (the summary records a hash of them)."""
+    import hashlib
+    import re
+    path = os.path.join(ROOT, "profiles", profile)
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    ratio = re.search(r"traffic_ratio: ([0-9.]+)", text)
+    digest = re.search(r"source_sha256: ([0-9a-f]+)", text)
+    if not ratio or not digest:
+        return None
+    h = hashlib.sha256()
+    for f in sources:
+        with open(os.path.join(ROOT, "paper_2608_08569_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return float(ratio.group(1)) if h.hexdigest()[:len(digest.group(1))] == digest.group(1) else None
+
+
 def peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -169,19 +189,14 @@ def decode_bytes(w, n_after):
     return w.layers * w.kv_heads * sum(per_b)
 
 
-def evict_bytes(w, n_before):
-    """Bytes an eviction must move, taking ordered compaction as the algorithm (Eq. 7-8): scores and
-    positions read once for the selection, then every kept row after the first evicted slot moved
-    (read and written: K, V, score, pos). The first evicted slot is at least the sink count, so
-    rows T..budget-M is the least that moves; this lower bound is what is counted."""
+def evict_bytes(w, n_before, moved_rows):
+    """Bytes an ordered in-place eviction must move (Eq. 7-8): each unit over budget reads its
+    scores and positions once for the selection (8 B per slot), and every kept row that changes
+    slot (all kept rows after the first evicted slot) is read and written with its K, V, score and
+    position. moved_rows[u] is counted from the positions before and after the eviction."""
     es = 2 if w.dtype == torch.bfloat16 else 4
     row = 2 * w.head_dim * es + 8
-    tot = 0
-    for n, bud in zip(n_before, w.budget):
-        if n <= bud:
-            continue
-        tot += 8 * n
-    return w.layers * w.kv_heads * tot
+    return int(8 * int(n_before.sum()) + 2 * row * int(moved_rows.sum()))
 
 
 # ----------------------------------------------------------------------------- GPU arm
@@ -203,9 +218,10 @@ class Runner:
         self.sess = Session(self.desc, w.budget, w.gamma, sink=w.sink, recent_frac=w.recent_frac, device=device)
         self.out = torch.empty(w.steps, w.layers, w.batch, w.q_heads, w.head_dim, dtype=w.dtype, device=device)
 
-    def request(self, timers=None, lengths=None):
-        """One request: stage 1, then every decode step with evictions. With `timers`, records a
-        CUDA event pair around every decode launch (on the launch stream)."""
+    def request(self, timers=None, lengths=None, evict_timers=None, moved=None):
+        """One request: stage 1, then every decode step with evictions. With `timers` (and
+        `evict_timers`), records a CUDA event pair around every decode (evict) launch on the launch
+        stream. With `moved`, records per eviction the units' lengths and moved rows (this syncs)."""
         w, s = self.w, self.sess
         s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
         n = s.cache["len"][:, 0, 0].tolist() if lengths is not None else None
@@ -226,7 +242,35 @@ class Runner:
                 if n is not None:
                     lengths.append(("evict", list(n)))
                     n = [min(x, b) for x, b in zip(n, w.budget)]
+                if moved is not None:
+                    pos_before = s.cache["pos"].clone()
+                    n_before = s.cache["len"].clone()
+                if evict_timers is not None:
+                    f0 = torch.cuda.Event(enable_timing=True)
+                    f1 = torch.cuda.Event(enable_timing=True)
+                    f0.record(stream)
                 s.evict()
+                if evict_timers is not None:
+                    f1.record(stream)
+                    evict_timers.append((f0, f1))
+                if moved is not None:
+                    moved.append(moved_rows(pos_before, n_before, s.cache["pos"], s.cache["len"]))
+
+
+def moved_rows(pos_before, n_before, pos_after, n_after):
+    """(lengths before, rows that changed slot) per unit of one eviction: a unit that shrank keeps
+    its rows up to the first slot whose position changed and moves every kept row after it."""
+    C = pos_before.shape[-1]
+    pb = pos_before.reshape(-1, C)
+    pa = pos_after.reshape(-1, C)
+    nb = n_before.reshape(-1).long()
+    na = n_after.reshape(-1).long()
+    idx = torch.arange(C, device=pb.device)
+    differs = (pb != pa) & (idx[None, :] < na[:, None])
+    first = torch.where(differs.any(1), differs.float().argmax(1), na)
+    shrank = na < nb
+    moved = torch.where(shrank, na - first, torch.zeros_like(na))
+    return nb[shrank].cpu().numpy(), moved.cpu().numpy()
 
 
 def gpu_arm(args, rank, world, local):
@@ -239,7 +283,7 @@ def gpu_arm(args, rank, world, local):
         r.request()
     torch.cuda.synchronize()
     barrier(world)
-    timers, lengths = [], []
+    timers, lengths, ev_timers = [], [], []
     with ClockSampler(local) as clk:
         torch.cuda.synchronize()
         barrier(world)
@@ -247,7 +291,7 @@ def gpu_arm(args, rank, world, local):
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record()
         for k in range(args.steps):
-            r.request(timers=timers, lengths=lengths if k == 0 else None)
+            r.request(timers=timers, lengths=lengths if k == 0 else None, evict_timers=ev_timers)
         e1.record()
         torch.cuda.synchronize()
         barrier(world)
@@ -265,15 +309,48 @@ def gpu_arm(args, rank, world, local):
     achieved = bytes_per_request * args.steps / (dec_ms / 1000.0) / 1e9
     peak, peak_kind = peaks()
     n_evict = w.steps // w.interval
+    tr = profiled_traffic_ratio("decode_mma_kernel_stress.md", ["decode_mma.cu", "ptx.cuh", "common.cuh"])
+    alg_per_launch = bytes_per_request / max(1, len(dec_lens))
     roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
-                "frac": round(achieved / peak, 4), "traffic": None,
-                "kernel": "decode_kernel (append + GQA attention + decayed score)",
+                "frac": round(achieved / peak, 4),
+                "traffic": None if tr is None or w.name != "stress" else int(tr * alg_per_launch),
+                "kernel": "decode_mma_kernel (append + GQA attention + decayed score)",
+                "traffic_source": "profiles/decode_mma_kernel_stress.md: dram bytes / algorithmic bytes on steady "
+                                  "launches, times this run's algorithmic bytes per launch",
                 "peak_source": f"{peak_kind} hbm_gbs",
                 "avg_launch_us": round(avg_ms * 1000.0, 2),
                 "alg_bytes_per_launch": int(bytes_per_request / max(1, len(dec_lens))),
                 "decode_share_of_step": round(dec_ms / ms, 4)}
+    # The same split at the first eviction: before it the cache holds the whole stage-1 output.
+    pre = [i for i in range(len(timers)) if i % w.steps < w.interval]
+    post = [i for i in range(len(timers)) if i % w.steps >= w.interval]
+    for name, ids in (("before_first_evict", pre), ("after_first_evict", post)):
+        b = sum(decode_bytes(w, dec_lens[i % w.steps]) for i in ids)
+        t = sum(timers[i][0].elapsed_time(timers[i][1]) for i in ids)
+        if t > 0:
+            roofline[f"achieved_{name}"] = round(b / (t / 1000.0) / 1e9, 1)
     # kernels per request: 3 stage-1 kernels, one decode launch per step, one evict per interval
     gpu_launches = args.steps * (3 + w.steps + n_evict)
+
+    # The eviction kernel against the same peak: bytes from an untimed replay of one request.
+    moved = []
+    r.request(moved=moved)
+    torch.cuda.synchronize()
+    ev_bytes = sum(evict_bytes(w, nb, mv) for nb, mv in moved)
+    ev_ms = sum(a.elapsed_time(b) for a, b in ev_timers)
+    if ev_timers and ev_ms > 0:
+        ev_ach = ev_bytes * args.steps / (ev_ms / 1000.0) / 1e9
+        etr = profiled_traffic_ratio("evict_kernel_stress.md", ["evict.cu", "common.cuh"])
+        roofline_evict = {"bound": "hbm", "achieved": round(ev_ach, 1), "peak": peak, "unit": "GB/s",
+                          "frac": round(ev_ach / peak, 4),
+                          "traffic": None if etr is None or w.name != "stress" else
+                          int(etr * ev_bytes / max(1, len(moved))),
+                          "kernel": "evict_kernel (top-N select + ordered in-place compaction)",
+                          "avg_launch_us": round(1000.0 * ev_ms / len(ev_timers), 2),
+                          "alg_bytes_per_launch": int(ev_bytes / max(1, len(moved))),
+                          "evict_share_of_step": round(ev_ms / ms, 4)}
+    else:
+        roofline_evict = None
 
     e2e = None
     if not args.no_e2e:
@@ -290,7 +367,8 @@ def gpu_arm(args, rank, world, local):
                    "gamma": w.gamma, "decode_steps_per_request": w.steps, "evict_interval": w.interval,
                    "parallelism": f"replicas x{world} (independent units, no collective)",
                    "l2": "inputs larger than L2 (decode reads ~0.9-7 GB per launch, L2 is 129 MB)"},
-        "roofline": roofline, "gpu_launches": gpu_launches, "clocks": clocks, "e2e": e2e,
+        "roofline": roofline, "roofline_evict": roofline_evict, "gpu_launches": gpu_launches, "clocks": clocks,
+        "e2e": e2e,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_sample(w, args.cpu_units)

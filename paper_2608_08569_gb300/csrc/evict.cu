@@ -1,24 +1,27 @@
 // Budgeted eviction of VoxZip (Sec. 3.2.2, Eq. 7-9): keep T sinks, the M most recent rows and
 // the top-N history rows by decayed score, then compact K, V, score and pos in place.
 //
-// One CTA per unit:
-//   select   an 8-pass MSB-first radix select over 64-bit keys (order-preserving score bits,
-//            then the complemented position, so equal scores rank the lower position higher)
-//            finds the key of the N-th best history row. Keys are unique within a unit, so
-//            "key >= threshold" keeps exactly N rows.
-//   compact  slots are scanned in order, 1024 at a time; a block scan gives every kept slot its
-//            destination (its rank among kept slots) and the rows move in sub-chunks of rank
-//            order. A kept row never moves up (dest <= src), and the rows of a sub-chunk are all
-//            read into shared memory before any is written, so no row is overwritten before it
-//            is read: later sub-chunks read only slots at or beyond their own ranks, which lie
-//            past every destination written earlier.
+// One CTA of 512 threads per unit:
+//   select   MSB-first radix select (4 passes of 8 bits) over an order-preserving 32-bit image of
+//            the history scores gives the N-th best score. Only when that score is tied and not all
+//            tied rows fit does a second select over their positions (ascending) run, so that
+//            equal scores keep the lower position. Positions within a unit are unique.
+//   compact  slots are scanned 512 at a time; a block scan gives each kept slot its rank, and the
+//            kept slots of up to kSegment ranks are listed in shared memory. Rows then move in
+//            rank order, kRows rows per sub-chunk, staged in registers with the loads of
+//            sub-chunk i+1 in flight while sub-chunk i is stored. A kept row never moves up
+//            (dest = rank <= src); sub-chunk i+1's sources sit at slots >= its ranks, beyond all
+//            of sub-chunk i's destinations, and the barrier after each sub-chunk's stores orders
+//            every load of sub-chunk i before any store of sub-chunk i+1, so no row is
+//            overwritten before it is read.
 #include "common.cuh"
 
 namespace voxzip {
 namespace {
 
-constexpr int kThreads = 1024;
-constexpr int kStageBytes = 32 * 1024;
+constexpr int kThreads = 512;
+constexpr int kSegment = 4096;   // ranks listed per compaction segment
+constexpr int kStageVecs = 2;    // 16-byte vectors per thread per sub-chunk (16 KB per CTA)
 
 struct EvictParams {
     void *k_cache, *v_cache;
@@ -30,15 +33,15 @@ struct EvictParams {
     float recent_frac;
 };
 
-__device__ __forceinline__ uint64_t order_key(float s, int32_t p) {
-    uint32_t b = __float_as_uint(s);
-    b = (b & 0x80000000u) ? ~b : (b | 0x80000000u);  // monotone map of fp32 order to uint32 order
-    return ((uint64_t)b << 32) | (uint64_t)(0xffffffffu - (uint32_t)p);
+__device__ __forceinline__ uint32_t score_key(float s) {  // monotone map of fp32 order to uint32 order
+    const uint32_t b = __float_as_uint(s);
+    return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
-// Block-wide exclusive scan of one int per thread (blockDim.x == kThreads).
+// Block-wide exclusive scan of one int per thread.
 __device__ int scan_excl(int v, int *total, int *warp_sums) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    constexpr int kWarps = kThreads / 32;
     int x = v;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -48,35 +51,90 @@ __device__ int scan_excl(int v, int *total, int *warp_sums) {
     if (lane == 31) warp_sums[warp] = x;
     __syncthreads();
     if (warp == 0) {
-        int s = warp_sums[lane];
+        int s = lane < kWarps ? warp_sums[lane] : 0;
 #pragma unroll
         for (int o = 1; o < 32; o <<= 1) {
             const int y = __shfl_up_sync(0xffffffffu, s, o);
             if (lane >= o) s += y;
         }
-        warp_sums[lane] = s;
+        if (lane < kWarps) warp_sums[lane] = s;
     }
     __syncthreads();
     const int r = (warp > 0 ? warp_sums[warp - 1] : 0) + x - v;
-    *total = warp_sums[31];
+    *total = warp_sums[kWarps - 1];
     __syncthreads();
     return r;
 }
 
+// One radix pass: histogram of digit (key >> shift) & 255 over the keys that match `prefix` above
+// the digit, then the digit holding the `rem`-th key counted from the top (descending = true) or
+// from the bottom. Updates prefix and rem; returns the count of keys equal to the final prefix
+// in the last pass (the bin size).
+struct RadixState {
+    uint32_t prefix;
+    int rem;
+    int bin;
+};
+
+template <bool kDescending, typename KeyFn>
+__device__ void radix_pass(int shift, int lo, int hi, KeyFn key_of, RadixState &st, unsigned *hist,
+                           RadixState *shared_st) {
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int i = tid; i < 256; i += kThreads) hist[i] = 0u;
+    __syncthreads();
+    const uint32_t mask_hi = shift == 24 ? 0u : (0xffffffffu << (shift + 8));
+    for (int j = lo + tid; j < hi; j += kThreads) {
+        bool valid;
+        const uint32_t k = key_of(j, valid);
+        if (valid && (k & mask_hi) == (st.prefix & mask_hi)) atomicAdd(&hist[(k >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (warp == 0) {
+        // Lane l holds 8 consecutive bins in scan order (from the top bin when descending).
+        unsigned c[8], s = 0;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            const int bin = kDescending ? 255 - (lane * 8 + k) : lane * 8 + k;
+            c[k] = hist[bin];
+            s += c[k];
+        }
+        unsigned incl = s;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const unsigned y = __shfl_up_sync(0xffffffffu, incl, o);
+            if (lane >= o) incl += y;
+        }
+        const unsigned excl = incl - s;
+        const bool hit = excl < (unsigned)st.rem && (unsigned)st.rem <= incl;
+        const unsigned ballot = __ballot_sync(0xffffffffu, hit);
+        if (lane == __ffs(ballot) - 1) {
+            unsigned cum = excl;
+            for (int k = 0; k < 8; ++k) {
+                if (cum + c[k] >= (unsigned)st.rem) {
+                    const int bin = kDescending ? 255 - (lane * 8 + k) : lane * 8 + k;
+                    shared_st->prefix = (st.prefix & mask_hi) | ((uint32_t)bin << shift);
+                    shared_st->rem = st.rem - (int)cum;
+                    shared_st->bin = (int)c[k];
+                    break;
+                }
+                cum += c[k];
+            }
+        }
+    }
+    __syncthreads();
+    st = *shared_st;
+}
+
 template <typename T, int D>
-__global__ void __launch_bounds__(kThreads) evict_kernel(const EvictParams p) {
-    constexpr int kVecPerRow = D * (int)sizeof(T) / 16;      // 16-byte vectors per K (or V) row
-    constexpr int kRowsPerStage = kStageBytes / (2 * D * (int)sizeof(T));
-    __shared__ uint4 stage[kStageBytes / 16];
-    __shared__ float stage_score[kRowsPerStage];
-    __shared__ int32_t stage_pos[kRowsPerStage];
-    __shared__ int32_t src_list[kThreads];
+__global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictParams p) {
+    constexpr int kVecPerRow = D * (int)sizeof(T) / 16;  // 16-byte vectors in one K (or V) row
+    constexpr int kRows = kThreads * kStageVecs / (2 * kVecPerRow);
+    __shared__ int32_t src_list[kSegment];
     __shared__ unsigned hist[256];
     __shared__ int warp_sums[32];
-    __shared__ unsigned long long sel_prefix;
-    __shared__ int sel_rem;
+    __shared__ RadixState shared_st;
 
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int tid = threadIdx.x;
     const UnitIdx ui = unit_of(blockIdx.x, p.B, p.L, p.Hkv, p.layer_begin);
     const int32_t n = p.len[ui.cache_unit];
     const int32_t bud = p.budget[ui.b];
@@ -98,107 +156,116 @@ __global__ void __launch_bounds__(kThreads) evict_kernel(const EvictParams p) {
     uint4 *vc = reinterpret_cast<uint4 *>(static_cast<T *>(p.v_cache) + ui.cache_unit * p.C * D);
     const int32_t c_end = n - M;  // history candidates are slots [T, c_end)
 
-    // Eq. 9: the key of the N-th largest candidate.
-    uint64_t prefix = 0;
-    int rem = N;
+    // Eq. 9: the N-th best history score, then (only if needed) the position cut among its ties.
+    uint32_t thr = 0u, pos_thr = 0xffffffffu;
+    bool all_ties = true;
     if (N > 0) {
-        for (int pass = 0; pass < 8; ++pass) {
-            const int shift = 56 - 8 * pass;
-            for (int i = tid; i < 256; i += kThreads) hist[i] = 0u;
-            __syncthreads();
-            for (int j = T_ + tid; j < c_end; j += kThreads) {
-                const uint64_t key = order_key(sc[j], ps[j]);
-                if (pass == 0 || (key >> (shift + 8)) == (prefix >> (shift + 8)))
-                    atomicAdd(&hist[(unsigned)(key >> shift) & 255u], 1u);
+        RadixState st{0u, N, 0};
+        auto skey = [&](int j, bool &valid) {
+            valid = true;
+            return score_key(sc[j]);
+        };
+        for (int shift = 24; shift >= 0; shift -= 8) radix_pass<true>(shift, T_, c_end, skey, st, hist, &shared_st);
+        thr = st.prefix;
+        all_ties = st.rem == st.bin;  // every candidate scoring exactly thr is kept
+        if (!all_ties) {
+            RadixState sp{0u, st.rem, 0};
+            auto pkey = [&](int j, bool &valid) {
+                valid = score_key(sc[j]) == thr;
+                return (uint32_t)ps[j];
+            };
+            for (int shift = 24; shift >= 0; shift -= 8)
+                radix_pass<false>(shift, T_, c_end, pkey, sp, hist, &shared_st);
+            pos_thr = sp.prefix;
+        }
+    }
+
+    // Eq. 7-8: ordered, in-place compaction of the kept rows.
+    int cursor = 0, rank0 = 0;
+    while (cursor < n) {
+        int seg = 0;
+        while (cursor < n && seg + kThreads <= kSegment) {
+            const int j = cursor + tid;
+            bool keep = false;
+            if (j < n) {
+                if (j < T_ || j >= c_end) {
+                    keep = true;
+                } else if (N > 0) {
+                    const uint32_t k = score_key(sc[j]);
+                    keep = k > thr || (k == thr && (all_ties || (uint32_t)ps[j] <= pos_thr));
+                }
             }
-            __syncthreads();
-            if (warp == 0) {
-                // Lane l holds bins 255-8l down to 248-8l: counts accumulate from the top bin.
-                const int top = 255 - lane * 8;
-                unsigned c[8], s = 0;
+            int total;
+            const int r = scan_excl(keep ? 1 : 0, &total, warp_sums);
+            if (keep) src_list[seg + r] = j;
+            seg += total;
+            cursor += kThreads;
+        }
+        __syncthreads();
+
+        // Move ranks [rank0, rank0 + seg) in sub-chunks of kRows, two sub-chunks in flight.
+        const int nsub = (seg + kRows - 1) / kRows;
+        uint4 buf[2][kStageVecs];
+        float bsc[2];
+        int32_t bps[2];
+        auto load_sub = [&](int s, uint4 (&b)[kStageVecs], float &bs, int32_t &bp) {
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    c[k] = hist[top - k];
-                    s += c[k];
-                }
-                unsigned incl = s;
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
-                    const unsigned y = __shfl_up_sync(0xffffffffu, incl, o);
-                    if (lane >= o) incl += y;
-                }
-                const unsigned excl = incl - s;
-                const bool hit = excl < (unsigned)rem && (unsigned)rem <= incl;
-                const unsigned ballot = __ballot_sync(0xffffffffu, hit);
-                if (lane == __ffs(ballot) - 1) {
-                    unsigned cum = excl;
-                    for (int k = 0; k < 8; ++k) {
-                        if (cum + c[k] >= (unsigned)rem) {
-                            sel_prefix = prefix | ((unsigned long long)(top - k) << shift);
-                            sel_rem = rem - (int)cum;
-                            break;
-                        }
-                        cum += c[k];
+            for (int k = 0; k < kStageVecs; ++k) {
+                const int v = tid + k * kThreads;
+                const int row = s * kRows + v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
+                if (row < seg) {
+                    const int src = src_list[row];
+                    if (src != rank0 + row) {
+                        const uint4 *from = w < kVecPerRow ? kc : vc;
+                        b[k] = from[(int64_t)src * kVecPerRow + (w % kVecPerRow)];
                     }
                 }
             }
-            __syncthreads();
-            prefix = sel_prefix;
-            rem = sel_rem;
-        }
-    }
-    const uint64_t thr = prefix;  // keys above thr are kept, plus the first `rem` equal to it
-
-    // Eq. 7-8: ordered, in-place compaction of the kept rows.
-    int base_rank = 0, eq_seen = 0;
-    for (int c0 = 0; c0 < n; c0 += kThreads) {
-        const int j = c0 + tid;
-        const bool in = j < n;
-        const bool cand = in && j >= T_ && j < c_end;
-        const uint64_t key = cand ? order_key(sc[j], ps[j]) : 0ull;
-        const bool eq = cand && N > 0 && key == thr;
-        int eq_total;
-        const int eq_rank = scan_excl(eq ? 1 : 0, &eq_total, warp_sums);
-        const bool keep = in && (!cand || (N > 0 && (key > thr || (eq && eq_seen + eq_rank < rem))));
-        int kept_total;
-        const int k_rank = scan_excl(keep ? 1 : 0, &kept_total, warp_sums);
-        if (keep) src_list[k_rank] = j;
-        eq_seen += eq_total;
-        __syncthreads();
-        for (int r0 = 0; r0 < kept_total; r0 += kRowsPerStage) {
-            const int rows = min(kRowsPerStage, kept_total - r0);
-            for (int v = tid; v < rows * 2 * kVecPerRow; v += kThreads) {
-                const int row = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
-                const int src = src_list[r0 + row], dst = base_rank + r0 + row;
-                if (src != dst) {
-                    const uint4 *from = w < kVecPerRow ? kc : vc;
-                    stage[v] = from[(int64_t)src * kVecPerRow + (w % kVecPerRow)];
+            const int row = s * kRows + tid;
+            if (tid < kRows && row < seg) {
+                const int src = src_list[row];
+                if (src != rank0 + row) {
+                    bs = sc[src];
+                    bp = ps[src];
                 }
             }
-            for (int row = tid; row < rows; row += kThreads) {
-                const int src = src_list[r0 + row];
-                stage_score[row] = sc[src];
-                stage_pos[row] = ps[src];
-            }
-            __syncthreads();
-            for (int v = tid; v < rows * 2 * kVecPerRow; v += kThreads) {
-                const int row = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
-                const int src = src_list[r0 + row], dst = base_rank + r0 + row;
-                if (src != dst) {
-                    uint4 *to = w < kVecPerRow ? kc : vc;
-                    to[(int64_t)dst * kVecPerRow + (w % kVecPerRow)] = stage[v];
+        };
+        auto store_sub = [&](int s, const uint4 (&b)[kStageVecs], float bs, int32_t bp) {
+#pragma unroll
+            for (int k = 0; k < kStageVecs; ++k) {
+                const int v = tid + k * kThreads;
+                const int row = s * kRows + v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
+                if (row < seg) {
+                    const int dst = rank0 + row;
+                    if (src_list[row] != dst) {
+                        uint4 *to = w < kVecPerRow ? kc : vc;
+                        to[(int64_t)dst * kVecPerRow + (w % kVecPerRow)] = b[k];
+                    }
                 }
             }
-            for (int row = tid; row < rows; row += kThreads) {
-                const int dst = base_rank + r0 + row;
-                sc[dst] = stage_score[row];
-                ps[dst] = stage_pos[row];
+            const int row = s * kRows + tid;
+            if (tid < kRows && row < seg) {
+                const int dst = rank0 + row;
+                if (src_list[row] != dst) {
+                    sc[dst] = bs;
+                    ps[dst] = bp;
+                }
             }
+        };
+        if (nsub > 0) load_sub(0, buf[0], bsc[0], bps[0]);
+        for (int s = 0; s < nsub; s += 2) {
+            if (s + 1 < nsub) load_sub(s + 1, buf[1], bsc[1], bps[1]);
+            store_sub(s, buf[0], bsc[0], bps[0]);
             __syncthreads();
+            if (s + 1 < nsub) {
+                if (s + 2 < nsub) load_sub(s + 2, buf[0], bsc[0], bps[0]);
+                store_sub(s + 1, buf[1], bsc[1], bps[1]);
+                __syncthreads();
+            }
         }
-        base_rank += kept_total;
+        rank0 += seg;
     }
-    if (tid == 0) p.len[ui.cache_unit] = base_rank;  // == budget
+    if (tid == 0) p.len[ui.cache_unit] = rank0;  // == budget
 }
 
 template <typename T, int D>
