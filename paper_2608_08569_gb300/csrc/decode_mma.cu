@@ -14,10 +14,10 @@
 // and normaliser: every CTA rewrites its tokens' scores as gamma * s + sum_h p_h / Z_h and
 // combines one slice of the G x D outputs from all CTAs' partials.
 #include <cooperative_groups.h>
-#include <cudaTypedefs.h>
 
 #include "common.cuh"
 #include "ptx.cuh"
+#include "tmap.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -27,9 +27,6 @@ namespace {
 #ifndef VOXZIP_DECODE_WARPS
 #define VOXZIP_DECODE_WARPS 4      // consumer warps per CTA (16 tokens of every tile each)
 #endif
-#ifndef VOXZIP_DECODE_STAGES
-#define VOXZIP_DECODE_STAGES 3     // depth of the shared-memory tile ring
-#endif
 #ifndef VOXZIP_DECODE_CTA_OVERHEAD
 #define VOXZIP_DECODE_CTA_OVERHEAD 384  // fixed cost of one CTA in the split model, in tokens streamed
 #endif
@@ -37,7 +34,6 @@ namespace {
 constexpr int kConsumerWarps = VOXZIP_DECODE_WARPS;
 constexpr int kThreads = (kConsumerWarps + 1) * 32;
 constexpr int kTile = 16 * kConsumerWarps;      // tokens per pipeline stage
-constexpr int kStages = VOXZIP_DECODE_STAGES;
 constexpr int kBoxCols = 64;                    // bf16 elements per TMA box row (128 bytes)
 constexpr int kBoxBytes = kTile * kBoxCols * 2;
 constexpr uint32_t kWaitLimit = 1u << 24;
@@ -56,7 +52,7 @@ struct MmaParams {
     float gamma, scale_log2;
 };
 
-template <int D, int NT>
+template <int D, int NT, int kStages>
 struct Layout {
     static constexpr int kHalves = D / 64;
     static constexpr int kGP = 8 * NT;                         // heads padded to the MMA's N
@@ -79,11 +75,11 @@ __device__ __forceinline__ uint32_t swz(int row, int chunk) {  // byte offset in
     return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
-template <int D, int NT>
+template <int D, int NT, int kStages>
 __global__ void __launch_bounds__(kThreads)
 decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                   const MmaParams p) {
-    using Lay = Layout<D, NT>;
+    using Lay = Layout<D, NT, kStages>;
     constexpr int GP = Lay::kGP;
     constexpr int kHalves = Lay::kHalves;
     constexpr int kKSteps = D / 16;
@@ -442,37 +438,28 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
 }
 
 // ---------------------------------------------------------------- host side
-PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (fn == nullptr) {
-        void *ptr = nullptr;
-        cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-                cudaSuccess &&
-            q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+template <int D_, int NT_, int NS_>
+struct Tag {
+    static constexpr int D = D_, NT = NT_, NS = NS_;
+};
+
+// Calls f(Tag<D, NT, NS>{}) for the runtime shape; the kernel is instantiated for D in {64, 128},
+// NT in {1, 2} (group <= 8 or <= 16) and a ring of NS in {3, 4} stages.
+template <typename F>
+auto dispatch(int D, int NT, int NS, F &&f) {
+    if (D == 128) {
+        if (NT == 1) return NS == 4 ? f(Tag<128, 1, 4>{}) : f(Tag<128, 1, 3>{});
+        return NS == 4 ? f(Tag<128, 2, 4>{}) : f(Tag<128, 2, 3>{});
     }
-    return fn;
+    if (NT == 1) return NS == 4 ? f(Tag<64, 1, 4>{}) : f(Tag<64, 1, 3>{});
+    return NS == 4 ? f(Tag<64, 2, 4>{}) : f(Tag<64, 2, 3>{});
 }
 
-// The whole cache as a 2-D [rows][D] bf16 tensor; boxes of kTile rows x 64 columns, 128B swizzle.
-bool make_map(CUtensorMap *map, void *base, int64_t rows, int D) {
-    auto enc = tensor_map_encoder();
-    if (!enc) return false;
-    cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)D * 2};
-    cuuint32_t box[2] = {(cuuint32_t)kBoxCols, (cuuint32_t)kTile};
-    cuuint32_t estr[2] = {1, 1};
-    return enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, base, dims, strides, box, estr,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
-template <int D, int NT>
+template <typename K>
 bool configure() {  // kernel attributes are per function; set once per process
     static bool done = false;
     if (!done) {
-        auto kern = decode_mma_kernel<D, NT>;
+        auto kern = decode_mma_kernel<K::D, K::NT, K::NS>;
         if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem) != cudaSuccess ||
             cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
             return false;
@@ -481,38 +468,38 @@ bool configure() {  // kernel attributes are per function; set once per process
     return true;
 }
 
-// Resident CTAs per SM for a given dynamic shared-memory size (cached: the candidates repeat).
-template <int D, int NT>
-int occupancy_t(size_t smem) {
-    thread_local size_t last_smem[8] = {};
-    thread_local int last_occ[8] = {};
-    thread_local int next = 0;
-    for (int i = 0; i < 8; ++i)
-        if (last_smem[i] == smem) return last_occ[i];
-    if (!configure<D, NT>()) return 0;
-    int occ = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, decode_mma_kernel<D, NT>, kThreads, smem) != cudaSuccess)
-        occ = 0;
-    last_smem[next] = smem;
-    last_occ[next] = occ;
-    next = (next + 1) % 8;
-    return occ;
+// How many clusters of S CTAs, each with `smem` bytes of shared memory, fit the GPU at once.
+template <typename K>
+int max_active_clusters(int S, size_t smem) {
+    if (!configure<K>()) return 0;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)S, 1024, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)S;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, decode_mma_kernel<K::D, K::NT, K::NS>, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return 0;
+    }
+    return n;
 }
 
-int occupancy(int D, int NT, size_t smem) {
-    if (D == 128) return NT == 1 ? occupancy_t<128, 1>(smem) : occupancy_t<128, 2>(smem);
-    return NT == 1 ? occupancy_t<64, 1>(smem) : occupancy_t<64, 2>(smem);
-}
-
-template <int D, int NT>
+template <typename K>
 cudaError_t launch_t(const CUtensorMap &tmk, const CUtensorMap &tmv, const MmaParams &prm, int S, int units,
                      cudaStream_t stream) {
-    auto kern = decode_mma_kernel<D, NT>;
-    if (!configure<D, NT>()) return cudaErrorInvalidValue;
+    auto kern = decode_mma_kernel<K::D, K::NT, K::NS>;
+    if (!configure<K>()) return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)S, (unsigned)units, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = Layout<D, NT>::bytes(prm.chunk_cap);
+    cfg.dynamicSmemBytes = Layout<K::D, K::NT, K::NS>::bytes(prm.chunk_cap);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -522,6 +509,46 @@ cudaError_t launch_t(const CUtensorMap &tmk, const CUtensorMap &tmv, const MmaPa
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, kern, tmk, tmv, prm);
+}
+
+struct Plan {
+    int S, NS, chunk_cap;
+};
+
+// Chooses the cluster size S and ring depth NS. For each S the CTAs hold ceil(nmax/S) tokens
+// (rounded up to a tile, which also keeps the set of shared-memory sizes small); the deeper ring
+// is taken when it does not reduce how many clusters are resident. The cost is the number of
+// cluster rounds over the units times (tokens per CTA + a fixed per-CTA overhead), plus one
+// round's worth of tail.
+Plan plan(int D, int NT, int units, int nmax) {
+    Plan best{0, 3, 0};
+    double best_cost = 0.0;
+    for (int S = 1; S <= kMaxCluster; S <<= 1) {
+        int cap = (nmax + S - 1) / S;
+        if (S > 1 && cap < kTile / 2) break;
+        cap = (cap + kTile - 1) / kTile * kTile;
+        int ns_best = 0, cl_best = 0;
+        for (int ns = 4; ns >= 3; --ns) {
+            const size_t sm = dispatch(D, NT, ns, [&](auto k) {
+                using K = decltype(k);
+                return Layout<K::D, K::NT, K::NS>::bytes(cap);
+            });
+            if (sm > kMaxSmem) continue;
+            const int cl = dispatch(D, NT, ns, [&](auto k) { return max_active_clusters<decltype(k)>(S, sm); });
+            if (cl > cl_best) {
+                cl_best = cl;
+                ns_best = ns;
+            }
+        }
+        if (cl_best == 0) continue;
+        const double per_cta = (double)cap + VOXZIP_DECODE_CTA_OVERHEAD;
+        const double cost = (double)units / cl_best * per_cta + per_cta;
+        if (best.S == 0 || cost < best_cost) {
+            best = Plan{S, ns_best, cap};
+            best_cost = cost;
+        }
+    }
+    return best;
 }
 
 }  // namespace
@@ -542,46 +569,36 @@ cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, i
     const int NT = G <= 8 ? 1 : 2;
     const int units = layer_count * d.batch * d.kv_heads;
     const int nmax = (max_len > 0 && max_len < d.capacity) ? max_len : d.capacity;
-    // Cluster size: for each candidate S, CTAs hold ceil(nmax/S) tokens; the occupancy API gives how
-    // many fit an SM with that much shared memory, and the cost is the number of CTA waves times
-    // (tokens per CTA + a fixed per-CTA overhead), plus one CTA's worth of tail.
-    int sms = 148;
-    {
-        int dev = 0;
-        if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    }
-    auto smem_of = [&](int cap) {
-        return d.head_dim == 128 ? (NT == 1 ? Layout<128, 1>::bytes(cap) : Layout<128, 2>::bytes(cap))
-                                 : (NT == 1 ? Layout<64, 1>::bytes(cap) : Layout<64, 2>::bytes(cap));
+    // Plans are cached per (head dim, group tiles, units, length bucket of one tile).
+    struct Entry {
+        int D, NT, units, bucket;
+        Plan p;
     };
-    int S = 0;
-    double best = 0.0;
-    for (int s = 1; s <= kMaxCluster; s <<= 1) {
-        const int cap = (nmax + s - 1) / s;
-        if (s > 1 && cap < kTile / 2) break;
-        const size_t sm = smem_of(cap);
-        if (sm > kMaxSmem) continue;
-        const int occ = occupancy(d.head_dim, NT, sm);
-        if (occ <= 0) continue;
-        const double per_cta = (double)cap + VOXZIP_DECODE_CTA_OVERHEAD;
-        const double cost = (double)units * s * per_cta / ((double)sms * occ) + per_cta;
-        if (S == 0 || cost < best) {
-            S = s;
-            best = cost;
+    thread_local Entry cache[16];
+    thread_local int cache_next = 0;
+    const int bucket = (nmax + kTile - 1) / kTile;
+    Plan pl{0, 0, 0};
+    for (const Entry &e : cache)
+        if (e.p.S != 0 && e.D == d.head_dim && e.NT == NT && e.units == units && e.bucket == bucket) pl = e.p;
+    if (pl.S == 0) {
+        pl = plan(d.head_dim, NT, units, bucket * kTile);
+        if (pl.S == 0) {
+            *unsupported = true;
+            return cudaSuccess;
         }
+        cache[cache_next] = Entry{d.head_dim, NT, units, bucket, pl};
+        cache_next = (cache_next + 1) % 16;
     }
-    if (S == 0) {
-        *unsupported = true;
-        return cudaSuccess;
-    }
-    const int chunk_cap = (nmax + S - 1) / S;
+    const int S = pl.S;
+    const int chunk_cap = pl.chunk_cap;
     const int64_t rows = (int64_t)d.batch * d.layers * d.kv_heads * d.capacity;
     thread_local void *cached_k = nullptr, *cached_v = nullptr;
     thread_local int64_t cached_rows = 0;
     thread_local int cached_d = 0;
     thread_local CUtensorMap tmk, tmv;
     if (cached_k != k_cache || cached_v != v_cache || cached_rows != rows || cached_d != d.head_dim) {
-        if (!make_map(&tmk, k_cache, rows, d.head_dim) || !make_map(&tmv, v_cache, rows, d.head_dim)) {
+        if (!make_cache_map(&tmk, k_cache, rows, d.head_dim, kTile) ||
+            !make_cache_map(&tmv, v_cache, rows, d.head_dim, kTile)) {
             cached_k = cached_v = nullptr;
             *unsupported = true;
             return cudaSuccess;
@@ -608,10 +625,8 @@ cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, i
     prm.gamma = gamma;
     const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)d.head_dim);
     prm.scale_log2 = scale * 1.4426950408889634f;  // log2(e): exp(x) = 2^(x log2 e)
-    if (d.head_dim == 128)
-        return NT == 1 ? launch_t<128, 1>(tmk, tmv, prm, S, units, stream)
-                       : launch_t<128, 2>(tmk, tmv, prm, S, units, stream);
-    return NT == 1 ? launch_t<64, 1>(tmk, tmv, prm, S, units, stream) : launch_t<64, 2>(tmk, tmv, prm, S, units, stream);
+    return dispatch(d.head_dim, NT, pl.NS,
+                    [&](auto k) { return launch_t<decltype(k)>(tmk, tmv, prm, S, units, stream); });
 }
 
 }  // namespace voxzip
