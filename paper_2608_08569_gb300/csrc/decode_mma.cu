@@ -48,7 +48,7 @@ struct MmaParams {
     int32_t *pos, *len;
     __nv_bfloat16 *out;
     int32_t *status;
-    int32_t B, L, Hq, Hkv, G, C, layer_begin, chunk_cap;
+    int32_t B, L, Hq, Hkv, G, C, layer_begin, chunk_cap, n_hint;
     float gamma, scale_log2;
 };
 
@@ -59,7 +59,8 @@ struct Layout {
     static constexpr int kStageBytes = kHalves * kBoxBytes;
     static constexpr int kStagesOff = 0;                       // the ring; reused for o_w afterwards
     static constexpr int kRingBytes = kStages * kStageBytes;
-    static_assert(kRingBytes >= kConsumerWarps * kGP * D * 4, "ring too small to hold the warp partials");
+    static constexpr int kOStride = D + 4;                     // padded row of the output partials
+    static_assert(kRingBytes >= kConsumerWarps * kGP * kOStride * 4, "ring too small to hold the warp partials");
     static constexpr int kBarOff = kRingBytes;                 // full[kStages], empty[kStages]
     static constexpr int kPbufOff = kBarOff + 2 * kStages * 8;
     static constexpr int kPbufBytes = kConsumerWarps * 16 * kGP * 2;
@@ -108,6 +109,14 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     float *s_old = lg + (size_t)p.chunk_cap * GP;               // [chunk_cap] scores before the step
 
     const UnitIdx ui = unit_of(blockIdx.y, p.B, p.L, p.Hkv, p.layer_begin);
+    // While this unit's length is read, pull the first tiles of the range the launch's length hint
+    // predicts into L2 (exact when the unit is as long as the hint; otherwise a few wasted KB).
+    if (warp == kConsumerWarps && lane == 0) {
+        const int est_j0 = rank * ((p.n_hint + S - 1) / S);
+        const int rows = min(kStages * kTile, p.C - est_j0);
+        if (rows > 0)
+            ptx::prefetch_l2(p.k_cache + (ui.cache_unit * p.C + est_j0) * D, (uint32_t)rows * D * 2);
+    }
     const int32_t n_old = p.len[ui.cache_unit];
     const int32_t n = n_old + 1;
     if (n_old < 0 || n > p.C) {  // the same decision in every CTA of the cluster
@@ -347,23 +356,25 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                 if (g == 0) z_w[warp * GP + nt * 8 + 2 * qd + j] = v;
             }
         asm volatile("bar.sync 1, %0;" ::"r"(kConsumerWarps * 32) : "memory");  // the ring is drained
-        float *ow = o_w + warp * GP * D;
+        constexpr int OS = Lay::kOStride;
+        float *ow = o_w + warp * GP * OS;
 #pragma unroll
         for (int i = 0; i < kKSteps; ++i)
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) {
                 const int d0 = i * 16 + g, h0 = nt * 8 + 2 * qd;
-                ow[h0 * D + d0] = oacc[i][nt][0];
-                ow[(h0 + 1) * D + d0] = oacc[i][nt][1];
-                ow[h0 * D + d0 + 8] = oacc[i][nt][2];
-                ow[(h0 + 1) * D + d0 + 8] = oacc[i][nt][3];
+                ow[h0 * OS + d0] = oacc[i][nt][0];
+                ow[(h0 + 1) * OS + d0] = oacc[i][nt][1];
+                ow[h0 * OS + d0 + 8] = oacc[i][nt][2];
+                ow[(h0 + 1) * OS + d0 + 8] = oacc[i][nt][3];
             }
         asm volatile("bar.sync 1, %0;" ::"r"(kConsumerWarps * 32) : "memory");
         for (int e = tid; e < GP * D; e += kConsumerWarps * 32) {
-            float v = o_w[e];
+            const int at = (e / D) * OS + e % D;
+            float v = o_w[at];
 #pragma unroll
-            for (int w = 1; w < kConsumerWarps; ++w) v += o_w[w * GP * D + e];
-            o_cta[e] = v;
+            for (int w = 1; w < kConsumerWarps; ++w) v += o_w[w * GP * OS + at];
+            o_cta[at] = v;
         }
         if (tid < GP) {
             float v = 0.f;
@@ -409,10 +420,16 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
             const int j = j0 + i;
             const float prev = (j == n - 1) ? 0.f : s_old[i];
             float add = 0.f;
-            const float *pr = lg + i * GP;
+            const float4 *pr = reinterpret_cast<const float4 *>(lg + i * GP);
 #pragma unroll
-            for (int h = 0; h < GP; ++h)
-                if (h < p.G) add += pr[h] * fac_self[h];
+            for (int h4 = 0; h4 < GP / 4; ++h4) {
+                const float4 v = pr[h4];
+                const int h = h4 * 4;
+                if (h < p.G) add += v.x * fac_self[h];
+                if (h + 1 < p.G) add += v.y * fac_self[h + 1];
+                if (h + 2 < p.G) add += v.z * fac_self[h + 2];
+                if (h + 3 < p.G) add += v.w * fac_self[h + 3];
+            }
             sc[j] = p.gamma * prev + add;
         }
     }
@@ -424,8 +441,9 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         for (int i = lo + tid; i < hi; i += kThreads) {
             const int h = i / D;
             float part[kMaxCluster];
+            const int at = h * Lay::kOStride + i % D;
 #pragma unroll
-            for (int r = 0; r < kMaxCluster; ++r) part[r] = r < S ? *cluster.map_shared_rank(&o_cta[i], r) : 0.f;
+            for (int r = 0; r < kMaxCluster; ++r) part[r] = r < S ? *cluster.map_shared_rank(&o_cta[at], r) : 0.f;
             float o = 0.f;
 #pragma unroll
             for (int r = 0; r < kMaxCluster; ++r)
@@ -621,7 +639,7 @@ cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, i
     prm.out = static_cast<__nv_bfloat16 *>(out);
     prm.status = status;
     prm.B = d.batch; prm.L = d.layers; prm.Hq = d.q_heads; prm.Hkv = d.kv_heads; prm.G = G;
-    prm.C = d.capacity; prm.layer_begin = layer_begin; prm.chunk_cap = chunk_cap;
+    prm.C = d.capacity; prm.layer_begin = layer_begin; prm.chunk_cap = chunk_cap; prm.n_hint = nmax;
     prm.gamma = gamma;
     const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)d.head_dim);
     prm.scale_log2 = scale * 1.4426950408889634f;  // log2(e): exp(x) = 2^(x log2 e)
