@@ -1,27 +1,28 @@
 // Budgeted eviction of VoxZip (Sec. 3.2.2, Eq. 7-9): keep T sinks, the M most recent rows and
 // the top-N history rows by decayed score, then compact K, V, score and pos in place.
 //
-// One CTA of 512 threads per unit:
+// One CTA of 256 threads per unit (small enough that every unit of a launch is resident at once):
 //   select   MSB-first radix select (4 passes of 8 bits) over an order-preserving 32-bit image of
 //            the history scores gives the N-th best score. Only when that score is tied and not all
 //            tied rows fit does a second select over their positions (ascending) run, so that
 //            equal scores keep the lower position. Positions within a unit are unique.
-//   compact  slots are scanned 512 at a time; a block scan gives each kept slot its rank, and the
+//   compact  slots are scanned 256 at a time; a block scan gives each kept slot its rank, and the
 //            kept slots of up to kSegment ranks are listed in shared memory. Rows then move in
-//            rank order, kRows rows per sub-chunk, staged in registers with the loads of
-//            sub-chunk i+1 in flight while sub-chunk i is stored. A kept row never moves up
-//            (dest = rank <= src); sub-chunk i+1's sources sit at slots >= its ranks, beyond all
-//            of sub-chunk i's destinations, and the barrier after each sub-chunk's stores orders
-//            every load of sub-chunk i before any store of sub-chunk i+1, so no row is
-//            overwritten before it is read.
+//            rank order, kRows rows per sub-chunk, through a kPipe-deep ring of shared-memory
+//            stages filled by cp.async: the loads of the next kPipe-1 sub-chunks are in flight
+//            while one is stored. A kept row never moves up (dest = rank <= src). Sources of a
+//            later sub-chunk sit at slots >= its ranks, beyond every destination of an earlier one,
+//            so in-flight loads never see a store; and a barrier after all of a sub-chunk's loads
+//            have landed precedes its stores, so no row is overwritten before it is read.
 #include "common.cuh"
 
 namespace voxzip {
 namespace {
 
-constexpr int kThreads = 512;
-constexpr int kSegment = 4096;   // ranks listed per compaction segment
-constexpr int kStageVecs = 2;    // 16-byte vectors per thread per sub-chunk (16 KB per CTA)
+constexpr int kThreads = 256;
+constexpr int kSegment = 1024;   // ranks listed per compaction segment
+constexpr int kStageVecs = 2;    // 16-byte vectors per thread per sub-chunk (8 KB per CTA)
+constexpr int kPipe = 3;         // sub-chunks in flight
 
 struct EvictParams {
     void *k_cache, *v_cache;
@@ -126,10 +127,13 @@ __device__ void radix_pass(int shift, int lo, int hi, KeyFn key_of, RadixState &
 }
 
 template <typename T, int D>
-__global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictParams p) {
+__global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p) {
     constexpr int kVecPerRow = D * (int)sizeof(T) / 16;  // 16-byte vectors in one K (or V) row
     constexpr int kRows = kThreads * kStageVecs / (2 * kVecPerRow);
     __shared__ int32_t src_list[kSegment];
+    __shared__ uint4 stage[kPipe][kThreads * kStageVecs];
+    __shared__ float stage_sc[kPipe][kRows];
+    __shared__ int32_t stage_ps[kPipe][kRows];
     __shared__ unsigned hist[256];
     __shared__ int warp_sums[32];
     __shared__ RadixState shared_st;
@@ -203,64 +207,72 @@ __global__ void __launch_bounds__(kThreads, 4) evict_kernel(const EvictParams p)
         }
         __syncthreads();
 
-        // Move ranks [rank0, rank0 + seg) in sub-chunks of kRows, two sub-chunks in flight.
+        // Move ranks [rank0, rank0 + seg) in sub-chunks of kRows through the cp.async ring.
         const int nsub = (seg + kRows - 1) / kRows;
-        uint4 buf[2][kStageVecs];
-        float bsc[2];
-        int32_t bps[2];
-        auto load_sub = [&](int s, uint4 (&b)[kStageVecs], float &bs, int32_t &bp) {
+        auto load_sub = [&](int sub) {
+            const int st = sub % kPipe;
 #pragma unroll
             for (int k = 0; k < kStageVecs; ++k) {
                 const int v = tid + k * kThreads;
-                const int row = s * kRows + v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
+                const int row = sub * kRows + v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
                 if (row < seg) {
                     const int src = src_list[row];
                     if (src != rank0 + row) {
-                        const uint4 *from = w < kVecPerRow ? kc : vc;
-                        b[k] = from[(int64_t)src * kVecPerRow + (w % kVecPerRow)];
+                        const uint4 *from = (w < kVecPerRow ? kc : vc) + (int64_t)src * kVecPerRow + (w % kVecPerRow);
+                        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
+                                         (uint32_t)__cvta_generic_to_shared(&stage[st][v])),
+                                     "l"(from)
+                                     : "memory");
                     }
                 }
             }
-            const int row = s * kRows + tid;
+            const int row = sub * kRows + tid;
             if (tid < kRows && row < seg) {
                 const int src = src_list[row];
                 if (src != rank0 + row) {
-                    bs = sc[src];
-                    bp = ps[src];
+                    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                                     (uint32_t)__cvta_generic_to_shared(&stage_sc[st][tid])),
+                                 "l"(sc + src)
+                                 : "memory");
+                    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(
+                                     (uint32_t)__cvta_generic_to_shared(&stage_ps[st][tid])),
+                                 "l"(ps + src)
+                                 : "memory");
                 }
             }
         };
-        auto store_sub = [&](int s, const uint4 (&b)[kStageVecs], float bs, int32_t bp) {
+        auto store_sub = [&](int sub) {
+            const int st = sub % kPipe;
 #pragma unroll
             for (int k = 0; k < kStageVecs; ++k) {
                 const int v = tid + k * kThreads;
-                const int row = s * kRows + v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
+                const int row = sub * kRows + v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
                 if (row < seg) {
                     const int dst = rank0 + row;
                     if (src_list[row] != dst) {
                         uint4 *to = w < kVecPerRow ? kc : vc;
-                        to[(int64_t)dst * kVecPerRow + (w % kVecPerRow)] = b[k];
+                        to[(int64_t)dst * kVecPerRow + (w % kVecPerRow)] = stage[st][v];
                     }
                 }
             }
-            const int row = s * kRows + tid;
+            const int row = sub * kRows + tid;
             if (tid < kRows && row < seg) {
                 const int dst = rank0 + row;
                 if (src_list[row] != dst) {
-                    sc[dst] = bs;
-                    ps[dst] = bp;
+                    sc[dst] = stage_sc[st][tid];
+                    ps[dst] = stage_ps[st][tid];
                 }
             }
         };
-        if (nsub > 0) load_sub(0, buf[0], bsc[0], bps[0]);
-        for (int s = 0; s < nsub; s += 2) {
-            if (s + 1 < nsub) load_sub(s + 1, buf[1], bsc[1], bps[1]);
-            store_sub(s, buf[0], bsc[0], bps[0]);
-            __syncthreads();
-            if (s + 1 < nsub) {
-                if (s + 2 < nsub) load_sub(s + 2, buf[0], bsc[0], bps[0]);
-                store_sub(s + 1, buf[1], bsc[1], bps[1]);
-                __syncthreads();
+        for (int it = 0; it < nsub + kPipe - 1; ++it) {
+            if (it < nsub) load_sub(it);
+            asm volatile("cp.async.commit_group;" ::: "memory");
+            const int sub = it - (kPipe - 1);
+            if (sub >= 0) {
+                asm volatile("cp.async.wait_group %0;" ::"n"(kPipe - 1) : "memory");
+                __syncthreads();  // every thread's loads of `sub` have landed
+                store_sub(sub);
+                __syncthreads();  // its stage is drained before the next refill
             }
         }
         rank0 += seg;
