@@ -27,8 +27,17 @@ namespace {
 #ifndef VOXZIP_DECODE_WARPS
 #define VOXZIP_DECODE_WARPS 4      // consumer warps per CTA (16 tokens of every tile each)
 #endif
-#ifndef VOXZIP_DECODE_CTA_OVERHEAD
-#define VOXZIP_DECODE_CTA_OVERHEAD 384  // fixed cost of one CTA in the split model, in tokens streamed
+#ifndef VOXZIP_DECODE_CTA_FIXED_US
+#define VOXZIP_DECODE_CTA_FIXED_US 5.0     // a CTA's fixed latency: first tiles, exchange, exit
+#endif
+#ifndef VOXZIP_DECODE_STAGE_TOKENS_PER_US
+#define VOXZIP_DECODE_STAGE_TOKENS_PER_US 20.0  // one CTA's streaming rate per ring stage in flight
+#endif
+#ifndef VOXZIP_DECODE_SM_TOKENS_PER_US
+#define VOXZIP_DECODE_SM_TOKENS_PER_US 90.0     // one SM's share of HBM bandwidth (~46 GB/s of K+V)
+#endif
+#ifndef VOXZIP_DECODE_GPU_TOKENS_PER_US
+#define VOXZIP_DECODE_GPU_TOKENS_PER_US 12000.0  // the whole GPU near HBM peak (~6.1 TB/s of K+V)
 #endif
 
 constexpr int kConsumerWarps = VOXZIP_DECODE_WARPS;
@@ -462,15 +471,22 @@ struct Tag {
 };
 
 // Calls f(Tag<D, NT, NS>{}) for the runtime shape; the kernel is instantiated for D in {64, 128},
-// NT in {1, 2} (group <= 8 or <= 16) and a ring of NS in {3, 4} stages.
+// NT in {1, 2} (group <= 8 or <= 16) and a ring of NS in {3, 4, 6, 8} stages.
+constexpr int kRingDepths[] = {3, 4, 6, 8};
+
+template <int D, int NT, typename F>
+auto dispatch_ns(int NS, F &&f) {
+    switch (NS) {
+        case 4: return f(Tag<D, NT, 4>{});
+        case 6: return f(Tag<D, NT, 6>{});
+        case 8: return f(Tag<D, NT, 8>{});
+        default: return f(Tag<D, NT, 3>{});
+    }
+}
 template <typename F>
 auto dispatch(int D, int NT, int NS, F &&f) {
-    if (D == 128) {
-        if (NT == 1) return NS == 4 ? f(Tag<128, 1, 4>{}) : f(Tag<128, 1, 3>{});
-        return NS == 4 ? f(Tag<128, 2, 4>{}) : f(Tag<128, 2, 3>{});
-    }
-    if (NT == 1) return NS == 4 ? f(Tag<64, 1, 4>{}) : f(Tag<64, 1, 3>{});
-    return NS == 4 ? f(Tag<64, 2, 4>{}) : f(Tag<64, 2, 3>{});
+    if (D == 128) return NT == 1 ? dispatch_ns<128, 1>(NS, f) : dispatch_ns<128, 2>(NS, f);
+    return NT == 1 ? dispatch_ns<64, 1>(NS, f) : dispatch_ns<64, 2>(NS, f);
 }
 
 template <typename K>
@@ -533,37 +549,42 @@ struct Plan {
     int S, NS, chunk_cap;
 };
 
-// Chooses the cluster size S and ring depth NS. For each S the CTAs hold ceil(nmax/S) tokens
-// (rounded up to a tile, which also keeps the set of shared-memory sizes small); the deeper ring
-// is taken when it does not reduce how many clusters are resident. The cost is the number of
-// cluster rounds over the units times (tokens per CTA + a fixed per-CTA overhead), plus one
-// round's worth of tail.
+// Chooses the cluster size S and ring depth NS with a time model. For each (S, NS) the CTAs hold
+// ceil(nmax/S) tokens (shared memory sized for that, rounded up to 16 tokens); the occupancy API
+// gives how many clusters are resident. Every resident cluster takes ceil(units / clusters) units
+// in turn; a unit costs a CTA's fixed latency plus its tokens at one CTA's streaming rate, which
+// grows with the ring stages in flight until the CTAs of an SM share its bandwidth; and no launch
+// beats the GPU's streaming rate.
 Plan plan(int D, int NT, int units, int nmax) {
     Plan best{0, 3, 0};
     double best_cost = 0.0;
+    int sms = 148;
+    {
+        int dev = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    }
+    const double total = (double)units * nmax;
     for (int S = 1; S <= kMaxCluster; S <<= 1) {
         int cap = (nmax + S - 1) / S;
         if (S > 1 && cap < kTile / 2) break;
-        cap = (cap + kTile - 1) / kTile * kTile;
-        int ns_best = 0, cl_best = 0;
-        for (int ns = 4; ns >= 3; --ns) {
+        cap = (cap + 15) / 16 * 16;
+        for (int ns : kRingDepths) {
             const size_t sm = dispatch(D, NT, ns, [&](auto k) {
                 using K = decltype(k);
                 return Layout<K::D, K::NT, K::NS>::bytes(cap);
             });
             if (sm > kMaxSmem) continue;
             const int cl = dispatch(D, NT, ns, [&](auto k) { return max_active_clusters<decltype(k)>(S, sm); });
-            if (cl > cl_best) {
-                cl_best = cl;
-                ns_best = ns;
+            if (cl <= 0) continue;
+            const double per_sm = fmax(1.0, (double)cl * S / sms);
+            const double rate = fmin(VOXZIP_DECODE_STAGE_TOKENS_PER_US * ns, VOXZIP_DECODE_SM_TOKENS_PER_US / per_sm);
+            const double rounds = (double)((units + cl - 1) / cl);
+            const double per_cta = VOXZIP_DECODE_CTA_FIXED_US + (double)((nmax + S - 1) / S) / rate;
+            const double cost = fmax(rounds * per_cta, total / VOXZIP_DECODE_GPU_TOKENS_PER_US);
+            if (best.S == 0 || cost < best_cost) {
+                best = Plan{S, ns, cap};
+                best_cost = cost;
             }
-        }
-        if (cl_best == 0) continue;
-        const double per_cta = (double)cap + VOXZIP_DECODE_CTA_OVERHEAD;
-        const double cost = (double)units / cl_best * per_cta + per_cta;
-        if (best.S == 0 || cost < best_cost) {
-            best = Plan{S, ns_best, cap};
-            best_cost = cost;
         }
     }
     return best;
