@@ -4,15 +4,18 @@
 // Grid: one thread-block cluster of S CTAs per (layer, sequence, kv-head) unit; CTA r owns the
 // token range [r*ceil(n/S), (r+1)*ceil(n/S)). Per CTA, one producer warp streams the range's K
 // tiles and then its V tiles (64 tokens each) with 2-D tensor-map TMA loads (128-byte swizzle)
-// into a 4-stage shared-memory ring guarded by mbarriers; four consumer warps take 16 tokens of
-// every tile:
+// into a shared-memory ring guarded by mbarriers; four consumer warps take 16 tokens of every tile:
 //   phase K  S = K_tile Q^T on the tensor cores (mma.sync m16n8k16, tokens as M, the group's
-//            query heads as N), scaled logits kept in shared memory, per-head CTA maximum;
-//   phase V  p = 2^(logit - max_cta), kept for the score update; O^T += V_tile^T P^T on the
-//            tensor cores with bf16 probabilities and fp32 accumulators; per-head sums.
-// One cluster exchange through distributed shared memory then gives the global per-head maximum
-// and normaliser: every CTA rewrites its tokens' scores as gamma * s + sum_h p_h / Z_h and
-// combines one slice of the G x D outputs from all CTAs' partials.
+//            query heads as N); scaled logits kept in shared memory; a running per-head maximum
+//            and normaliser (online softmax statistics).
+//   phase V p = 2^(logit - max_cta); O^T += V_tile^T P^T on the tensor cores. A CTA that holds the
+//            whole unit (S = 1) already has the final statistics: it rewrites the scores tile by
+//            tile as gamma * s + sum_h p_h / Z_h. In a cluster p is kept in shared memory instead.
+// In a cluster, one exchange through distributed shared memory then gives the unit's per-head
+// maximum and normaliser: every CTA rewrites its tokens' scores and combines one slice of the
+// G x D outputs from all CTAs' partials. (Exchanging the statistics between the two phases instead
+// makes every CTA wait twice for the slowest one of its cluster, which measured slower.)
+// The appended row is patched into its tile in shared memory, so no load waits for its store.
 #include <cooperative_groups.h>
 
 #include "common.cuh"
@@ -28,7 +31,10 @@ namespace {
 #define VOXZIP_DECODE_WARPS 4      // consumer warps per CTA (16 tokens of every tile each)
 #endif
 #ifndef VOXZIP_DECODE_CTA_FIXED_US
-#define VOXZIP_DECODE_CTA_FIXED_US 5.0     // a CTA's fixed latency: first tiles, exchange, exit
+#define VOXZIP_DECODE_CTA_FIXED_US 5.0     // a CTA's fixed latency: first tiles, exit
+#endif
+#ifndef VOXZIP_DECODE_CLUSTER_FIXED_US
+#define VOXZIP_DECODE_CLUSTER_FIXED_US 0.0  // added by the cluster exchange (S > 1)
 #endif
 #ifndef VOXZIP_DECODE_STAGE_TOKENS_PER_US
 #define VOXZIP_DECODE_STAGE_TOKENS_PER_US 20.0  // one CTA's streaming rate per ring stage in flight
@@ -73,8 +79,8 @@ struct Layout {
     static constexpr int kBarOff = kRingBytes;                 // full[kStages], empty[kStages]
     static constexpr int kPbufOff = kBarOff + 2 * kStages * 8;
     static constexpr int kPbufBytes = kConsumerWarps * 16 * kGP * 2;
-    static constexpr int kStatOff = kPbufOff + kPbufBytes;     // m_w[warps][kGP], z_w[warps][kGP], m_cta, z_cta, fac
-    static constexpr int kStatFloats = (2 * kConsumerWarps + 3) * kGP + kMaxCluster * kGP;
+    static constexpr int kStatOff = kPbufOff + kPbufBytes;     // m_w, z_w [warps][kGP]; m_cta, z_cta [kGP]; fac [S][kGP]
+    static constexpr int kStatFloats = (2 * kConsumerWarps + 2 + kMaxCluster) * kGP;
     static constexpr int kLgOff = kStatOff + kStatFloats * 4;  // logits / p [chunk_cap][kGP] fp32, then old scores
     static size_t bytes(int chunk_cap) {
         return 1024 + (size_t)kLgOff + (size_t)chunk_cap * kGP * 4 + (size_t)chunk_cap * 4;
@@ -85,7 +91,8 @@ __device__ __forceinline__ uint32_t swz(int row, int chunk) {  // byte offset in
     return (uint32_t)(row * 128 + ((chunk ^ (row & 7)) << 4));
 }
 
-template <int D, int NT, int kStages>
+// kCluster: launched in clusters of S > 1 CTAs (else one CTA holds the whole unit).
+template <int D, int NT, int kStages, bool kCluster>
 __global__ void __launch_bounds__(kThreads)
 decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                   const MmaParams p) {
@@ -97,6 +104,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     cg::cluster_group cluster = cg::this_cluster();
     const int S = (int)cluster.num_blocks();
     const int rank = (int)cluster.block_rank();
+    constexpr bool clustered = kCluster;
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     const int g = lane >> 2, qd = lane & 3;
 
@@ -110,21 +118,41 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     float *o_cta = o_w;                                        // the sum over warps lands in warp 0's slot
     float *m_w = reinterpret_cast<float *>(smem + Lay::kStatOff);
     float *z_w = m_w + kConsumerWarps * GP;
-    float *m_cta = z_w + kConsumerWarps * GP;
-    float *z_cta = m_cta + GP;
-    float *fac_self = z_cta + GP;
-    float *fac_all = fac_self + GP;                            // [kMaxCluster][GP]
+    float *m_cta = z_w + kConsumerWarps * GP;                  // this CTA's per-head maximum (log2 units)
+    float *z_cta = m_cta + GP;                                 // and normaliser relative to it
+    float *fac = z_cta + GP;                                   // [S][GP]: 2^(m_r - m) / Z; 0 for padding heads
     float *lg = reinterpret_cast<float *>(smem + Lay::kLgOff);
     float *s_old = lg + (size_t)p.chunk_cap * GP;               // [chunk_cap] scores before the step
 
     const UnitIdx ui = unit_of(blockIdx.y, p.B, p.L, p.Hkv, p.layer_begin);
+    const int64_t act_row = (int64_t)ui.l_local * p.B + ui.b;
+    const int64_t row_base = ui.cache_unit * p.C;
     // While this unit's length is read, pull the first tiles of the range the launch's length hint
     // predicts into L2 (exact when the unit is as long as the hint; otherwise a few wasted KB).
     if (warp == kConsumerWarps && lane == 0) {
         const int est_j0 = rank * ((p.n_hint + S - 1) / S);
         const int rows = min(kStages * kTile, p.C - est_j0);
-        if (rows > 0)
-            ptx::prefetch_l2(p.k_cache + (ui.cache_unit * p.C + est_j0) * D, (uint32_t)rows * D * 2);
+        if (rows > 0) ptx::prefetch_l2(p.k_cache + (row_base + est_j0) * D, (uint32_t)rows * D * 2);
+    }
+    // The queries do not depend on the length: load them first. Q^T is the B operand:
+    // b0b1 = Q[head][16ks + 2qd .. +1], b2b3 = Q[head][16ks + 8 + 2qd .. +1].
+    uint32_t qb[NT][kKSteps][2];
+    if (warp < kConsumerWarps) {
+        const __nv_bfloat16 *qg = p.q + (act_row * p.Hq + (int64_t)ui.h * p.G) * D;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+            const int head = nt * 8 + g;
+#pragma unroll
+            for (int ks = 0; ks < kKSteps; ++ks) {
+                if (head < p.G) {
+                    qb[nt][ks][0] = *reinterpret_cast<const uint32_t *>(qg + head * D + ks * 16 + 2 * qd);
+                    qb[nt][ks][1] = *reinterpret_cast<const uint32_t *>(qg + head * D + ks * 16 + 8 + 2 * qd);
+                } else {
+                    qb[nt][ks][0] = 0u;
+                    qb[nt][ks][1] = 0u;
+                }
+            }
+        }
     }
     const int32_t n_old = p.len[ui.cache_unit];
     const int32_t n = n_old + 1;
@@ -140,18 +168,24 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     const int j0 = min(n, rank * chunk);
     const int cnt = min(n, j0 + chunk) - j0;
     const int ntiles = (cnt + kTile - 1) / kTile;
-    const int64_t act_row = (int64_t)ui.l_local * p.B + ui.b;
-    const int64_t row_base = ui.cache_unit * p.C;
 
-    // Eq. 1: the CTA owning slot n-1 writes the new row; the fence orders these generic-proxy
-    // writes before the async-proxy (TMA) reads issued after the barrier below.
-    if (j0 <= n - 1 && n - 1 < j0 + cnt && tid < D / 4) {
-        const int64_t src = (act_row * p.Hkv + ui.h) * D + tid * 4;
-        const int64_t dst = (row_base + n - 1) * D + tid * 4;
-        *reinterpret_cast<uint2 *>(p.k_cache + dst) = *reinterpret_cast<const uint2 *>(p.k_new + src);
-        *reinterpret_cast<uint2 *>(p.v_cache + dst) = *reinterpret_cast<const uint2 *>(p.v_new + src);
-        if (tid == 0) p.pos[row_base + n - 1] = p.new_pos[ui.b];
-        asm volatile("fence.proxy.async.global;" ::: "memory");
+    // Eq. 1: the appended row is local row jn of the CTA whose range holds slot n-1. The consumer
+    // warp that owns that row of its tile keeps k_new / v_new in registers, stores them to the cache
+    // for later steps and writes them over the row the TMA brought in, so no load waits for the store.
+    const int jn = n - 1 - j0;
+    const bool own_new = jn >= 0 && jn < cnt;
+    const int t_new = own_new ? jn / kTile : -1;
+    const bool patcher = own_new && warp == (jn % kTile) / 16;
+    const uint32_t patch_off = own_new ? (uint32_t)(lane >> 3) * kBoxBytes + swz(jn % kTile, lane & 7) : 0u;
+    uint4 kn4 = make_uint4(0u, 0u, 0u, 0u), vn4 = make_uint4(0u, 0u, 0u, 0u);
+    if (patcher && lane < D / 8) {
+        const int64_t src = (act_row * p.Hkv + ui.h) * D + lane * 8;
+        kn4 = *reinterpret_cast<const uint4 *>(p.k_new + src);
+        vn4 = *reinterpret_cast<const uint4 *>(p.v_new + src);
+        const int64_t dst = (row_base + n - 1) * D + lane * 8;
+        *reinterpret_cast<uint4 *>(p.k_cache + dst) = kn4;
+        *reinterpret_cast<uint4 *>(p.v_cache + dst) = vn4;
+        if (lane == 0) p.pos[row_base + n - 1] = p.new_pos[ui.b];
     }
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
@@ -192,29 +226,13 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                     ptx::tma_load_2d(dst + h * kBoxBytes, is_k ? &tmk : &tmv, h * kBoxCols, y, &full[s]);
             }
         }
-        __syncwarp();  // reconverge the producer warp before the block-wide barrier
+        __syncwarp();  // reconverge the producer warp
     } else {
         // ------------------------------------------------------------- consumers
-        // Q^T as the B operand: b0b1 = Q[head][16ks + 2qd .. +1], b2b3 = Q[head][16ks + 8 + 2qd .. +1].
-        uint32_t qb[NT][kKSteps][2];
-        const __nv_bfloat16 *qg = p.q + (act_row * p.Hq + (int64_t)ui.h * p.G) * D;
+        // Running maximum and normaliser of this thread's logits, per head slot (nt, j).
+        float mx[NT][2], zx[NT][2];
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-            const int head = nt * 8 + g;
-#pragma unroll
-            for (int ks = 0; ks < kKSteps; ++ks) {
-                if (head < p.G) {
-                    qb[nt][ks][0] = *reinterpret_cast<const uint32_t *>(qg + head * D + ks * 16 + 2 * qd);
-                    qb[nt][ks][1] = *reinterpret_cast<const uint32_t *>(qg + head * D + ks * 16 + 8 + 2 * qd);
-                } else {
-                    qb[nt][ks][0] = 0u;
-                    qb[nt][ks][1] = 0u;
-                }
-            }
-        }
-        float mx[NT][2];
-#pragma unroll
-        for (int nt = 0; nt < NT; ++nt) mx[nt][0] = mx[nt][1] = -INFINITY;
+        for (int nt = 0; nt < NT; ++nt) mx[nt][0] = mx[nt][1] = -INFINITY, zx[nt][0] = zx[nt][1] = 0.f;
         const int r0 = warp * 16;
 
         // Phase K: logits of this warp's 16 tokens of every tile.
@@ -226,7 +244,13 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
             }
             const int lt0 = t * kTile + r0;
             if (lt0 < cnt) {
-                const uint32_t base = ptx::smem_u32(stages + s * Lay::kStageBytes);
+                uint8_t *stage = stages + s * Lay::kStageBytes;
+                const bool patch = patcher && t == t_new;
+                if (patch) {
+                    if (lane < D / 8) *reinterpret_cast<uint4 *>(stage + patch_off) = kn4;
+                    __syncwarp();
+                }
+                const uint32_t base = ptx::smem_u32(stage);
                 float acc[NT][4];
 #pragma unroll
                 for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
@@ -242,56 +266,86 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                             ptx::mma_bf16_16816(acc[nt], a0, a1, a2, a3, qb[nt][h * 4 + kk][0], qb[nt][h * 4 + kk][1]);
                     }
                 }
+                // acc[nt][2 * half + j]: token lt0 + g + 8 * half, head nt * 8 + 2 * qd + j.
+                const bool va = lt0 + g < cnt, vb = lt0 + g + 8 < cnt;
 #pragma unroll
-                for (int half = 0; half < 2; ++half) {
-                    const int lt = lt0 + g + half * 8;
-                    const bool valid = lt < cnt;
+                for (int nt = 0; nt < NT; ++nt) {
+                    float la[2], lb[2];
 #pragma unroll
-                    for (int nt = 0; nt < NT; ++nt) {
-                        const float l0 = valid ? acc[nt][half * 2] * p.scale_log2 : -INFINITY;
-                        const float l1 = valid ? acc[nt][half * 2 + 1] * p.scale_log2 : -INFINITY;
-                        mx[nt][0] = fmaxf(mx[nt][0], l0);
-                        mx[nt][1] = fmaxf(mx[nt][1], l1);
-                        if (valid) *reinterpret_cast<float2 *>(lg + lt * GP + nt * 8 + 2 * qd) = make_float2(l0, l1);
+                    for (int j = 0; j < 2; ++j) {
+                        la[j] = va ? acc[nt][j] * p.scale_log2 : -INFINITY;
+                        lb[j] = vb ? acc[nt][2 + j] * p.scale_log2 : -INFINITY;
+                        const float m_new = fmaxf(mx[nt][j], fmaxf(la[j], lb[j]));
+                        // The normaliser is needed before phase V only without a cluster; keeping it
+                        // off the per-tile path otherwise matters when one CTA fills an SM.
+                        if (!clustered && m_new != -INFINITY)
+                            zx[nt][j] = zx[nt][j] * exp2f(mx[nt][j] - m_new) + exp2f(la[j] - m_new) +
+                                        exp2f(lb[j] - m_new);
+                        mx[nt][j] = m_new;
                     }
+                    if (va) *reinterpret_cast<float2 *>(lg + (lt0 + g) * GP + nt * 8 + 2 * qd) = make_float2(la[0], la[1]);
+                    if (vb)
+                        *reinterpret_cast<float2 *>(lg + (lt0 + g + 8) * GP + nt * 8 + 2 * qd) = make_float2(lb[0], lb[1]);
                 }
+                if (patch) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");  // before the slot's next TMA
             }
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&empty[s]);
         }
-        // CTA maximum per head.
+        // Per-head statistics of the warp (merge over the 8 lanes that share qd), then of the CTA.
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
             for (int j = 0; j < 2; ++j) {
-                float v = mx[nt][j];
-                v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 4));
-                v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 8));
-                v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, 16));
-                if (g == 0) m_w[warp * GP + nt * 8 + 2 * qd + j] = v;
+                float m = mx[nt][j], z = zx[nt][j];
+#pragma unroll
+                for (int off = 4; off <= 16; off <<= 1) {
+                    const float mo = __shfl_xor_sync(0xffffffffu, m, off);
+                    const float zo = __shfl_xor_sync(0xffffffffu, z, off);
+                    const float mm = fmaxf(m, mo);
+                    z = (m == -INFINITY ? 0.f : z * exp2f(m - mm)) + (mo == -INFINITY ? 0.f : zo * exp2f(mo - mm));
+                    m = mm;
+                }
+                if (g == 0) {
+                    m_w[warp * GP + nt * 8 + 2 * qd + j] = m;
+                    z_w[warp * GP + nt * 8 + 2 * qd + j] = z;
+                }
             }
+        asm volatile("cp.async.wait_all;" ::: "memory");  // this thread's old scores have landed
         asm volatile("bar.sync 1, %0;" ::"r"(kConsumerWarps * 32) : "memory");
         if (tid < GP) {
-            float v = -INFINITY;
-            for (int w = 0; w < kConsumerWarps; ++w) v = fmaxf(v, m_w[w * GP + tid]);
-            m_cta[tid] = v;
+            float m = -INFINITY, z = 0.f;
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) m = fmaxf(m, m_w[w * GP + tid]);
+#pragma unroll
+            for (int w = 0; w < kConsumerWarps; ++w) {
+                const float mw = m_w[w * GP + tid];
+                if (mw != -INFINITY) z += z_w[w * GP + tid] * exp2f(mw - m);
+            }
+            m_cta[tid] = m;
+            z_cta[tid] = z;
         }
+        // A CTA that holds the whole unit has its final statistics now.
+        if (!clustered && tid < GP) fac[tid] = tid < p.G ? 1.f / z_cta[tid] : 0.f;
         asm volatile("bar.sync 1, %0;" ::"r"(kConsumerWarps * 32) : "memory");
 
-        // Phase V: probabilities with the CTA maximum, P V on the tensor cores.
+        // Phase V: probabilities with the CTA maximum, P V on the tensor cores; without a cluster
+        // also the score update (Eq. 6), else p is kept for it.
         float oacc[kKSteps][NT][4];
 #pragma unroll
         for (int i = 0; i < kKSteps; ++i)
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) oacc[i][nt][0] = oacc[i][nt][1] = oacc[i][nt][2] = oacc[i][nt][3] = 0.f;
-        float zs[NT][2];
-        float mc[NT][2];
+        float mc[NT][2], rc[NT][2], zv[NT][2];
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) {
-            zs[nt][0] = zs[nt][1] = 0.f;
-            mc[nt][0] = m_cta[nt * 8 + 2 * qd];
-            mc[nt][1] = m_cta[nt * 8 + 2 * qd + 1];
-        }
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+            for (int j = 0; j < 2; ++j) {
+                mc[nt][j] = m_cta[nt * 8 + 2 * qd + j];
+                rc[nt][j] = clustered ? 0.f : fac[nt * 8 + 2 * qd + j];
+                zv[nt][j] = 0.f;
+            }
+        float *sc = p.score + row_base + j0;
         for (int t = 0; t < ntiles && ok; ++t) {
             const int i = ntiles + t, s = i % kStages;
             if (!__all_sync(0xffffffffu, ptx::mbar_wait_bounded(&full[s], (i / kStages) & 1, kWaitLimit))) {
@@ -305,22 +359,33 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                 for (int half = 0; half < 2; ++half) {
                     const int lt = lt0 + g + half * 8;
                     const bool valid = lt < cnt;
+                    float add = 0.f;
 #pragma unroll
                     for (int nt = 0; nt < NT; ++nt) {
                         float p0 = 0.f, p1 = 0.f;
                         if (valid) {
-                            float2 l = *reinterpret_cast<float2 *>(lg + lt * GP + nt * 8 + 2 * qd);
+                            const float2 l = *reinterpret_cast<const float2 *>(lg + lt * GP + nt * 8 + 2 * qd);
                             p0 = exp2f(l.x - mc[nt][0]);
                             p1 = exp2f(l.y - mc[nt][1]);
-                            *reinterpret_cast<float2 *>(lg + lt * GP + nt * 8 + 2 * qd) = make_float2(p0, p1);
+                            if (clustered) {
+                                *reinterpret_cast<float2 *>(lg + lt * GP + nt * 8 + 2 * qd) = make_float2(p0, p1);
+                                zv[nt][0] += p0;
+                                zv[nt][1] += p1;
+                            } else {
+                                add += p0 * rc[nt][0] + p1 * rc[nt][1];
+                            }
                         }
-                        zs[nt][0] += p0;
-                        zs[nt][1] += p1;
                         *reinterpret_cast<uint32_t *>(pbuf + (g + half * 8) * GP * 2 + (nt * 8 + 2 * qd) * 2) =
                             ptx::pack_bf16(p0, p1);
                     }
+                    if (!clustered) {  // Eq. 6: A = gamma * [A, 0] + sum over the heads (a token's four lanes)
+                        add += __shfl_xor_sync(0xffffffffu, add, 1);
+                        add += __shfl_xor_sync(0xffffffffu, add, 2);
+                        if (valid && qd == 0) sc[lt] = lt == jn ? add : p.gamma * s_old[lt] + add;
+                    }
                 }
                 // Rows past the range may hold anything; zero them so 0 * garbage cannot be NaN.
+                bool wrote = false;
                 if (lt0 + 16 > cnt) {
                     for (int e = lane; e < 16 * kHalves * 8; e += 32) {
                         const int row = e / (kHalves * 8), rest = e % (kHalves * 8);
@@ -328,8 +393,13 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                             *reinterpret_cast<uint4 *>(stage + (rest >> 3) * kBoxBytes + swz(r0 + row, rest & 7)) =
                                 make_uint4(0u, 0u, 0u, 0u);
                     }
-                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    wrote = true;
                 }
+                if (patcher && t == t_new) {
+                    if (lane < D / 8) *reinterpret_cast<uint4 *>(stage + patch_off) = vn4;
+                    wrote = true;
+                }
+                if (wrote) asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
                 __syncwarp();
                 uint32_t pb[NT][2];
 #pragma unroll
@@ -353,17 +423,19 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&empty[s]);
         }
-        // Per-head sums and partial outputs of this warp, then of the CTA (fixed summation order).
+        if (clustered) {  // per-head sums of the warp, then of the CTA (fixed order)
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt)
+            for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-            for (int j = 0; j < 2; ++j) {
-                float v = zs[nt][j];
-                v += __shfl_xor_sync(0xffffffffu, v, 4);
-                v += __shfl_xor_sync(0xffffffffu, v, 8);
-                v += __shfl_xor_sync(0xffffffffu, v, 16);
-                if (g == 0) z_w[warp * GP + nt * 8 + 2 * qd + j] = v;
-            }
+                for (int j = 0; j < 2; ++j) {
+                    float v = zv[nt][j];
+                    v += __shfl_xor_sync(0xffffffffu, v, 4);
+                    v += __shfl_xor_sync(0xffffffffu, v, 8);
+                    v += __shfl_xor_sync(0xffffffffu, v, 16);
+                    if (g == 0) z_w[warp * GP + nt * 8 + 2 * qd + j] = v;
+                }
+        }
+        // Partial outputs of this warp, then of the CTA (fixed summation order).
         asm volatile("bar.sync 1, %0;" ::"r"(kConsumerWarps * 32) : "memory");  // the ring is drained
         constexpr int OS = Lay::kOStride;
         float *ow = o_w + warp * GP * OS;
@@ -385,82 +457,78 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
             for (int w = 1; w < kConsumerWarps; ++w) v += o_w[w * GP * OS + at];
             o_cta[at] = v;
         }
-        if (tid < GP) {
+        if (clustered && tid < GP) {
             float v = 0.f;
 #pragma unroll
             for (int w = 0; w < kConsumerWarps; ++w) v += z_w[w * GP + tid];
             z_cta[tid] = v;
         }
-        asm volatile("cp.async.wait_all;" ::: "memory");
     }
     if (!ok) raise_status(p.status, VOXZIP_DEV_TIMEOUT);
     __syncthreads();
-    cluster.sync();  // every CTA's m_cta, z_cta, o_cta are final
-
-    // Global per-head maximum and normaliser; fac_all[r][h] = 2^(m_r - m) / Z.
-    if (tid < GP) {
-        float mr[kMaxCluster], zr[kMaxCluster];
+    if (clustered) {
+        cluster.sync();  // every CTA's m_cta, z_cta, o_cta are final
+        // The unit's per-head maximum m and normaliser Z; fac[r][h] = 2^(m_r - m) / Z.
+        if (tid < GP) {
+            float mr[kMaxCluster], zr[kMaxCluster];
 #pragma unroll
-        for (int r = 0; r < kMaxCluster; ++r) {
-            mr[r] = r < S ? *cluster.map_shared_rank(&m_cta[tid], r) : -INFINITY;
-            zr[r] = r < S ? *cluster.map_shared_rank(&z_cta[tid], r) : 0.f;
+            for (int r = 0; r < kMaxCluster; ++r) {
+                mr[r] = r < S ? *cluster.map_shared_rank(&m_cta[tid], r) : -INFINITY;
+                zr[r] = r < S ? *cluster.map_shared_rank(&z_cta[tid], r) : 0.f;
+            }
+            float m = -INFINITY;
+#pragma unroll
+            for (int r = 0; r < kMaxCluster; ++r) m = fmaxf(m, mr[r]);
+            float z = 0.f;
+#pragma unroll
+            for (int r = 0; r < kMaxCluster; ++r) {
+                mr[r] = mr[r] == -INFINITY ? 0.f : exp2f(mr[r] - m);
+                z += mr[r] * zr[r];
+            }
+            const float rzv = tid < p.G ? 1.f / z : 0.f;
+#pragma unroll
+            for (int r = 0; r < kMaxCluster; ++r)
+                if (r < S) fac[r * GP + tid] = mr[r] * rzv;
         }
-        float m = -INFINITY;
-#pragma unroll
-        for (int r = 0; r < kMaxCluster; ++r) m = fmaxf(m, mr[r]);
-        float z = 0.f;
-#pragma unroll
-        for (int r = 0; r < kMaxCluster; ++r) {
-            mr[r] = mr[r] == -INFINITY ? 0.f : exp2f(mr[r] - m);
-            z += mr[r] * zr[r];
-        }
-        const float rz = 1.f / z;
-#pragma unroll
-        for (int r = 0; r < kMaxCluster; ++r)
-            if (r < S) fac_all[r * GP + tid] = mr[r] * rz;
-        fac_self[tid] = fac_all[rank * GP + tid];
-    }
-    __syncthreads();
-
-    // Eq. 6 for this CTA's tokens: A = gamma * [A, 0] + sum over the group's heads.
-    {
-        float *sc = p.score + row_base;
+        __syncthreads();
+        // Eq. 6 for this CTA's tokens: A = gamma * [A, 0] + sum over the group's heads.
+        const float *fs = fac + rank * GP;
+        float *sc = p.score + row_base + j0;
         for (int i = tid; i < cnt; i += kThreads) {
-            const int j = j0 + i;
-            const float prev = (j == n - 1) ? 0.f : s_old[i];
             float add = 0.f;
             const float4 *pr = reinterpret_cast<const float4 *>(lg + i * GP);
 #pragma unroll
             for (int h4 = 0; h4 < GP / 4; ++h4) {
                 const float4 v = pr[h4];
-                const int h = h4 * 4;
-                if (h < p.G) add += v.x * fac_self[h];
-                if (h + 1 < p.G) add += v.y * fac_self[h + 1];
-                if (h + 2 < p.G) add += v.z * fac_self[h + 2];
-                if (h + 3 < p.G) add += v.w * fac_self[h + 3];
+                add += v.x * fs[h4 * 4] + v.y * fs[h4 * 4 + 1] + v.z * fs[h4 * 4 + 2] + v.w * fs[h4 * 4 + 3];
             }
-            sc[j] = p.gamma * prev + add;
+            sc[i] = i == jn ? add : p.gamma * s_old[i] + add;
         }
     }
-    // Combine the partial outputs; CTA r writes slice r of the G x D outputs.
+    // Sum the CTAs' partial outputs, normalised; CTA r writes slice r of the G x D outputs.
     {
         const int total = p.G * D, per = (total + S - 1) / S;
         const int lo = rank * per, hi = min(total, lo + per);
         __nv_bfloat16 *og = p.out + (act_row * p.Hq + (int64_t)ui.h * p.G) * D;
         for (int i = lo + tid; i < hi; i += kThreads) {
             const int h = i / D;
-            float part[kMaxCluster];
             const int at = h * Lay::kOStride + i % D;
+            float o;
+            if (clustered) {
+                float part[kMaxCluster];
 #pragma unroll
-            for (int r = 0; r < kMaxCluster; ++r) part[r] = r < S ? *cluster.map_shared_rank(&o_cta[at], r) : 0.f;
-            float o = 0.f;
+                for (int r = 0; r < kMaxCluster; ++r) part[r] = r < S ? *cluster.map_shared_rank(&o_cta[at], r) : 0.f;
+                o = 0.f;
 #pragma unroll
-            for (int r = 0; r < kMaxCluster; ++r)
-                if (r < S) o += fac_all[r * GP + h] * part[r];
+                for (int r = 0; r < kMaxCluster; ++r)
+                    if (r < S) o += fac[r * GP + h] * part[r];
+            } else {
+                o = o_cta[at] * fac[h];
+            }
             og[i] = __float2bfloat16_rn(o);
         }
     }
-    cluster.sync();  // no CTA leaves while others may still read its shared memory
+    if (clustered) cluster.sync();  // no CTA leaves while others may still read its shared memory
     if (rank == 0 && tid == 0) p.len[ui.cache_unit] = n;
 }
 
@@ -489,14 +557,21 @@ auto dispatch(int D, int NT, int NS, F &&f) {
     return NT == 1 ? dispatch_ns<64, 1>(NS, f) : dispatch_ns<64, 2>(NS, f);
 }
 
+using KernelFn = void (*)(CUtensorMap, CUtensorMap, MmaParams);
+
+template <typename K>
+KernelFn kernel_for(int S) {
+    return S > 1 ? decode_mma_kernel<K::D, K::NT, K::NS, true> : decode_mma_kernel<K::D, K::NT, K::NS, false>;
+}
+
 template <typename K>
 bool configure() {  // kernel attributes are per function; set once per process
     static bool done = false;
     if (!done) {
-        auto kern = decode_mma_kernel<K::D, K::NT, K::NS>;
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem) != cudaSuccess ||
-            cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
-            return false;
+        for (KernelFn kern : {kernel_for<K>(1), kernel_for<K>(2)})
+            if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem) != cudaSuccess ||
+                cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
+                return false;
         done = true;
     }
     return true;
@@ -518,7 +593,7 @@ int max_active_clusters(int S, size_t smem) {
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     int n = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, decode_mma_kernel<K::D, K::NT, K::NS>, &cfg) != cudaSuccess) {
+    if (cudaOccupancyMaxActiveClusters(&n, kernel_for<K>(S), &cfg) != cudaSuccess) {
         cudaGetLastError();
         return 0;
     }
@@ -528,7 +603,7 @@ int max_active_clusters(int S, size_t smem) {
 template <typename K>
 cudaError_t launch_t(const CUtensorMap &tmk, const CUtensorMap &tmv, const MmaParams &prm, int S, int units,
                      cudaStream_t stream) {
-    auto kern = decode_mma_kernel<K::D, K::NT, K::NS>;
+    const KernelFn kern = kernel_for<K>(S);
     if (!configure<K>()) return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)S, (unsigned)units, 1);
@@ -549,13 +624,20 @@ struct Plan {
     int S, NS, chunk_cap;
 };
 
+struct PlanModel {
+    double cta_fixed_us, cluster_fixed_us, stage_tokens_per_us, sm_tokens_per_us, gpu_tokens_per_us;
+};
+constexpr PlanModel kPlanModel{VOXZIP_DECODE_CTA_FIXED_US, VOXZIP_DECODE_CLUSTER_FIXED_US,
+                               VOXZIP_DECODE_STAGE_TOKENS_PER_US, VOXZIP_DECODE_SM_TOKENS_PER_US,
+                               VOXZIP_DECODE_GPU_TOKENS_PER_US};
+
 // Chooses the cluster size S and ring depth NS with a time model. For each (S, NS) the CTAs hold
 // ceil(nmax/S) tokens (shared memory sized for that, rounded up to 16 tokens); the occupancy API
 // gives how many clusters are resident. Every resident cluster takes ceil(units / clusters) units
-// in turn; a unit costs a CTA's fixed latency plus its tokens at one CTA's streaming rate, which
-// grows with the ring stages in flight until the CTAs of an SM share its bandwidth; and no launch
-// beats the GPU's streaming rate.
-Plan plan(int D, int NT, int units, int nmax) {
+// in turn; a unit costs a CTA's fixed latency (more with a cluster exchange) plus its tokens at one
+// CTA's streaming rate, which grows with the ring stages in flight until the CTAs resident on an SM
+// share its bandwidth; and no launch beats the GPU's streaming rate.
+Plan plan(int D, int NT, int units, int nmax, const PlanModel &md = kPlanModel) {
     Plan best{0, 3, 0};
     double best_cost = 0.0;
     int sms = 148;
@@ -576,11 +658,12 @@ Plan plan(int D, int NT, int units, int nmax) {
             if (sm > kMaxSmem) continue;
             const int cl = dispatch(D, NT, ns, [&](auto k) { return max_active_clusters<decltype(k)>(S, sm); });
             if (cl <= 0) continue;
-            const double per_sm = fmax(1.0, (double)cl * S / sms);
-            const double rate = fmin(VOXZIP_DECODE_STAGE_TOKENS_PER_US * ns, VOXZIP_DECODE_SM_TOKENS_PER_US / per_sm);
+            const double per_sm = fmax(1.0, (double)min(units, cl) * S / sms);  // CTAs sharing an SM
+            const double rate = fmin(md.stage_tokens_per_us * ns, md.sm_tokens_per_us / per_sm);
             const double rounds = (double)((units + cl - 1) / cl);
-            const double per_cta = VOXZIP_DECODE_CTA_FIXED_US + (double)((nmax + S - 1) / S) / rate;
-            const double cost = fmax(rounds * per_cta, total / VOXZIP_DECODE_GPU_TOKENS_PER_US);
+            const double per_cta = md.cta_fixed_us + (S > 1 ? md.cluster_fixed_us : 0.0) +
+                                   (double)((nmax + S - 1) / S) / rate;
+            const double cost = fmax(rounds * per_cta, total / md.gpu_tokens_per_us);
             if (best.S == 0 || cost < best_cost) {
                 best = Plan{S, ns, cap};
                 best_cost = cost;
