@@ -94,6 +94,10 @@ class Oracle:
         lib = ctypes.CDLL(path)
         lib.vzo_stage1.argtypes = [_i32, _i32, _i32, _i32, _I32P, _I32P, _I32P, _i32, _F64P, _F64P,
                                    _i32, _i32, _F64P, _F64P, _I32P, _I32P, _I32P]
+        lib.vzo_stage1_ex.argtypes = [_i32, _i32, _i32, _i32, _I32P, _I32P, _I32P, _i32, _F64P, _F64P,
+                                      _i32, _i32, _i32, _F64P, _F64P, _I32P, _I32P, _I32P]
+        lib.vzo_segments_to_spans.argtypes = [_i32, _F64P, _F64P, _F64P, _I32P, _f64, _i32, _i32, _f64,
+                                              _I32P, _I32P, _I32P, _I32P, _I32P]
         lib.vzo_decode_step.argtypes = [_i32, _i32, _i32, _I32P, _F64P, _F64P, _F64P, _I32P, _F64P,
                                         _F64P, _F64P, _i32, _f64, _f64, _F64P]
         lib.vzo_evict.argtypes = [_i32, _I32P, _i32, _i32, _f32, _F64P, _F64P, _F64P, _I32P,
@@ -103,14 +107,17 @@ class Oracle:
                                      _F64P, _I32P, _f64, _f64, _i32, _i32, _i32, _f32, _F64P,
                                      _F64P, _I32P, _I32P, _F64P, _F64P, _F64P, _F64P, _I32P,
                                      _I32P, _I32P, _I32P]
-        for f in (lib.vzo_stage1, lib.vzo_decode_step, lib.vzo_evict, lib.vzo_run_unit):
+        for f in (lib.vzo_stage1, lib.vzo_stage1_ex, lib.vzo_segments_to_spans, lib.vzo_decode_step,
+                  lib.vzo_evict, lib.vzo_run_unit):
             f.restype = ctypes.c_int
         self.lib = lib
         self.path = path
 
     def stage1(self, x, in_len, audio_begin, audio_len, span_start, span_end, span_groups, *,
-               anchor=None, cache_is_bf16=False, capacity=None):
-        """Stage-1 fusion of one unit's rows. Returns dict(exact, stored, pos, slot_map, n)."""
+               anchor=None, cache_is_bf16=False, capacity=None, keep_background=True):
+        """Stage-1 fusion of one unit's rows (or of one sequence's embeddings). With
+        keep_background=False the audio no span covers is dropped (the "Partial" ablation) and
+        its tokens map to slot -1. Returns dict(exact, stored, pos, slot_map, n)."""
         x = _f64a(x)
         D = x.shape[1]
         ss, se, sg = _i32a(span_start), _i32a(span_end), _i32a(span_groups)
@@ -121,16 +128,41 @@ class Oracle:
         slot_map = np.full(max(int(in_len), 1), -1, np.int32)
         n = np.zeros(1, np.int32)
         anc = None if anchor is None else _f64a(anchor)
-        rc = self.lib.vzo_stage1(int(in_len), int(audio_begin), int(audio_len), len(ss),
-                                 _p(ss, _I32P), _p(se, _I32P), _p(sg, _I32P), D, _p(x, _F64P),
-                                 _p(anc, _F64P), int(bool(cache_is_bf16)), cap, _p(exact, _F64P),
-                                 _p(stored, _F64P), _p(pos, _I32P), _p(slot_map, _I32P),
-                                 _p(n, _I32P))
+        if keep_background:
+            rc = self.lib.vzo_stage1(int(in_len), int(audio_begin), int(audio_len), len(ss),
+                                     _p(ss, _I32P), _p(se, _I32P), _p(sg, _I32P), D, _p(x, _F64P),
+                                     _p(anc, _F64P), int(bool(cache_is_bf16)), cap, _p(exact, _F64P),
+                                     _p(stored, _F64P), _p(pos, _I32P), _p(slot_map, _I32P),
+                                     _p(n, _I32P))
+        else:
+            rc = self.lib.vzo_stage1_ex(int(in_len), int(audio_begin), int(audio_len), len(ss),
+                                        _p(ss, _I32P), _p(se, _I32P), _p(sg, _I32P), D, _p(x, _F64P),
+                                        _p(anc, _F64P), int(bool(cache_is_bf16)), 0, cap,
+                                        _p(exact, _F64P), _p(stored, _F64P), _p(pos, _I32P),
+                                        _p(slot_map, _I32P), _p(n, _I32P))
         if rc != OK:
             raise OracleError("vzo_stage1", rc)
         k = int(n[0])
         return dict(exact=exact[:k], stored=stored[:k], pos=pos[:k],
                     slot_map=slot_map[:int(in_len)], n=k)
+
+    def segments_to_spans(self, t_start, t_end, confidence, text_len, tau_total: float, audio_len: int,
+                          audio_begin: int = 0, threshold: float = 0.3):
+        """ASR segments -> token-index spans (confidence filter, Eq. 3). Returns
+        dict(start, end, groups, seg_index) as int32 arrays, one entry per kept segment."""
+        ts, te, cf = _f64a(t_start), _f64a(t_end), _f64a(confidence)
+        tl = _i32a(text_len)
+        n = len(ts)
+        assert len(te) == n and len(cf) == n and len(tl) == n
+        out = [np.zeros(max(n, 1), np.int32) for _ in range(4)]
+        k = np.zeros(1, np.int32)
+        rc = self.lib.vzo_segments_to_spans(n, _p(ts, _F64P), _p(te, _F64P), _p(cf, _F64P), _p(tl, _I32P),
+                                            float(tau_total), int(audio_len), int(audio_begin), float(threshold),
+                                            *[_p(a, _I32P) for a in out], _p(k, _I32P))
+        if rc != OK:
+            raise OracleError("vzo_segments_to_spans", rc)
+        m = int(k[0])
+        return dict(start=out[0][:m], end=out[1][:m], groups=out[2][:m], seg_index=out[3][:m])
 
     def decode_step(self, cache: UnitCache, q, k_new, v_new, new_pos: int, gamma: float,
                     scale: float):
@@ -226,6 +258,10 @@ def default() -> Oracle:
 
 def stage1(*a, **k):
     return default().stage1(*a, **k)
+
+
+def segments_to_spans(*a, **k):
+    return default().segments_to_spans(*a, **k)
 
 
 def decode_step(*a, **k):

@@ -9,9 +9,14 @@
  * a time, in the order the paper states its steps, with no blocking or fusion.
  *
  * Functions and the passages they follow:
+ *   vzo_segments_to_spans  Sec. 3.2.1: the confidence filter on ASR segments (keep those above
+ *                    the threshold, 0.3 in the paper) and the time-to-token-index map of Eq. 3.
  *   vzo_stage1       Sec. 3.2.1: semantic intervals given as token-index spans (Eq. 3 already
  *                    applied), uniform grouping + average pooling (Eq. 4), anchor addition,
  *                    background preservation and chronological concatenation (Eq. 5).
+ *   vzo_stage1_ex    the same with the background optional: the "T+A (Partial)" configuration
+ *                    of the stage-1 ablation (Sec. 4, Table of fusion strategies) drops the
+ *                    audio no semantic interval covers.
  *   vzo_decode_step  Sec. 3.1: cache append (Eq. 1) and scaled dot-product attention (Eq. 2);
  *                    Sec. 3.2.2: temporally decayed accumulated score (Eq. 6).
  *   vzo_evict        Sec. 3.2.2: T attention sinks, a recent window of 20 % of the budget,
@@ -22,8 +27,14 @@
  * hand-worked fixtures); none is "parity unpinned".
  *
  * Readings where the paper is silent (each is listed in the design notes):
- *   - stage 1 acts on each layer's prefilled K and V rows; the anchor term is an optional
- *     caller-supplied row per (span, group), zero when absent;
+ *   - "a confidence score above a threshold" is strict (confidence > threshold);
+ *   - Eq. 3 is evaluated as floor(L_a * (tau / tau_total)) in double, in that order; indices
+ *     are clamped to [0, L_a]; a segment that would start before the previous kept one ends
+ *     starts where that one ends (an empty interval if nothing is left); segments must come
+ *     sorted by start time;
+ *   - stage 1 acts on each layer's prefilled K and V rows (or on embeddings, the paper's own
+ *     setting); the anchor term is an optional caller-supplied row per (span, group), zero
+ *     when absent;
  *   - group j of a span of length l with g = min(n_groups, l) groups covers
  *     [s + floor(j*l/g), s + floor((j+1)*l/g)); empty spans yield nothing;
  *   - the slot of a fused group records the index of the group's first token as its position;
@@ -81,11 +92,11 @@ static double bf16_round(float f)
  *   slot_map   [in_len]      output slot of every input token
  * Returns VZO_OK, VZO_EINVAL for malformed spans, VZO_ECAPACITY if the output exceeds capacity.
  */
-int vzo_stage1(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t n_spans,
-               const int32_t *span_start, const int32_t *span_end, const int32_t *span_groups,
-               int32_t D, const double *x, const double *anchor, int32_t cache_is_bf16,
-               int32_t capacity, double *out_exact, double *out_stored, int32_t *pos,
-               int32_t *slot_map, int32_t *out_len)
+int vzo_stage1_ex(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t n_spans,
+                  const int32_t *span_start, const int32_t *span_end, const int32_t *span_groups,
+                  int32_t D, const double *x, const double *anchor, int32_t cache_is_bf16,
+                  int32_t keep_background, int32_t capacity, double *out_exact,
+                  double *out_stored, int32_t *pos, int32_t *slot_map, int32_t *out_len)
 {
     if (in_len < 0 || audio_begin < 0 || audio_len < 0 || D <= 0 || capacity < 0 ||
         (int64_t)audio_begin + audio_len > in_len || n_spans < 0)
@@ -144,6 +155,10 @@ int vzo_stage1(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t n
             t = span_end[i];
             anchor_row += span_groups[i];
             ++i;
+        } else if (!keep_background && t >= audio_begin && t < audio_begin + audio_len) {
+            /* "Partial": a background acoustic token is discarded; it maps to no slot. */
+            slot_map[t] = -1;
+            ++t;
         } else {
             /* Background audio or text token: preserved unchanged, in chronological order (Eq. 5). */
             if (slot >= capacity)
@@ -159,6 +174,71 @@ int vzo_stage1(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t n
         }
     }
     *out_len = slot;
+    return VZO_OK;
+}
+
+/* Stage 1 as the paper's main method runs it: background acoustic intervals preserved. */
+int vzo_stage1(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t n_spans,
+               const int32_t *span_start, const int32_t *span_end, const int32_t *span_groups,
+               int32_t D, const double *x, const double *anchor, int32_t cache_is_bf16,
+               int32_t capacity, double *out_exact, double *out_stored, int32_t *pos,
+               int32_t *slot_map, int32_t *out_len)
+{
+    return vzo_stage1_ex(in_len, audio_begin, audio_len, n_spans, span_start, span_end,
+                         span_groups, D, x, anchor, cache_is_bf16, 1, capacity, out_exact,
+                         out_stored, pos, slot_map, out_len);
+}
+
+/*
+ * The semantic set of one sequence (Sec. 3.2.1): ASR segments (start time, end time, text of
+ * L_t tokens, confidence) become token-index spans of the audio region.
+ *
+ *   t_start, t_end, confidence, text_len   [n_seg] per segment, sorted by t_start
+ *   tau_total   duration of the audio, seconds (> 0)
+ *   La          number of audio tokens; audio_begin = index of the first one in the prompt
+ *   threshold   a segment is kept when its confidence is above it
+ * Outputs, one entry per kept segment, in order:
+ *   span_start, span_end   [audio_begin + idx_start, audio_begin + idx_end) (Eq. 3)
+ *   span_groups            L_t of the segment
+ *   seg_index              which input segment it came from
+ *   n_spans                how many were kept
+ * Returns VZO_EINVAL for unsorted segments, t_end < t_start, L_t < 1 or tau_total <= 0.
+ */
+int vzo_segments_to_spans(int32_t n_seg, const double *t_start, const double *t_end,
+                          const double *confidence, const int32_t *text_len, double tau_total,
+                          int32_t La, int32_t audio_begin, double threshold, int32_t *span_start,
+                          int32_t *span_end, int32_t *span_groups, int32_t *seg_index,
+                          int32_t *n_spans)
+{
+    if (n_seg < 0 || !(tau_total > 0.0) || La < 0 || audio_begin < 0)
+        return VZO_EINVAL;
+    for (int32_t i = 0; i < n_seg; ++i) {
+        if (!(t_end[i] >= t_start[i]) || text_len[i] < 1 || (i > 0 && t_start[i] < t_start[i - 1]))
+            return VZO_EINVAL;
+    }
+    int32_t kept = 0;
+    int64_t prev_end = 0;
+    for (int32_t i = 0; i < n_seg; ++i) {
+        /* Keep only segments whose confidence is above the threshold. */
+        if (!(confidence[i] > threshold))
+            continue;
+        /* Eq. 3: idx = floor(L_a * (tau / tau_total)). */
+        double fs = floor((double)La * (t_start[i] / tau_total));
+        double fe = floor((double)La * (t_end[i] / tau_total));
+        int64_t s = fs < 0.0 ? 0 : (fs > (double)La ? La : (int64_t)fs);
+        int64_t e = fe < 0.0 ? 0 : (fe > (double)La ? La : (int64_t)fe);
+        if (s < prev_end)
+            s = prev_end;
+        if (e < s)
+            e = s;
+        span_start[kept] = (int32_t)(audio_begin + s);
+        span_end[kept] = (int32_t)(audio_begin + e);
+        span_groups[kept] = text_len[i];
+        seg_index[kept] = i;
+        prev_end = e;
+        ++kept;
+    }
+    *n_spans = kept;
     return VZO_OK;
 }
 

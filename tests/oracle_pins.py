@@ -172,6 +172,104 @@ def pin_stage1_structure(orc):
     np.testing.assert_allclose(r["exact"][0], row, rtol=1e-15)
 
 
+def pin_stage1_partial_hand(orc):
+    """Hand-worked "Partial" stage 1: the same example with the background audio dropped."""
+    g = _golden("stage1_hand.json")
+    x = np.array([[t, t * t] for t in range(g["in_len"])], float)
+    r = orc.stage1(x, g["in_len"], g["audio_begin"], g["audio_len"], g["span_start"], g["span_end"],
+                   g["span_groups"], keep_background=False)
+    p = g["partial"]
+    assert r["n"] == len(p["expected_rows"])
+    np.testing.assert_allclose(r["exact"], _rows(p["expected_rows"]), rtol=0, atol=1e-12)
+    np.testing.assert_array_equal(r["pos"], p["expected_pos"])
+    np.testing.assert_array_equal(r["slot_map"], p["expected_slot_map"])
+
+
+def pin_stage1_partial_relation(orc):
+    """Dropping the background removes exactly the background rows of the full stage 1 and
+    nothing else: the remaining rows, positions and their order are the full result's."""
+    rng = np.random.default_rng(5)
+    for trial in range(20):
+        in_len = int(rng.integers(1, 80))
+        ab = int(rng.integers(0, in_len))
+        al = int(rng.integers(0, in_len - ab + 1))
+        ss, se, sg = _random_spans(rng, ab, al)
+        x = _bf16(rng.standard_normal((in_len, 4)))
+        anchor = _bf16(rng.standard_normal((max(1, sum(sg)), 4)))
+        full = orc.stage1(x, in_len, ab, al, ss, se, sg, anchor=anchor, cache_is_bf16=True)
+        part = orc.stage1(x, in_len, ab, al, ss, se, sg, anchor=anchor, cache_is_bf16=True,
+                          keep_background=False)
+        inside = np.zeros(in_len, bool)
+        for s, e in zip(ss, se):
+            inside[s:e] = True
+        background = np.zeros(in_len, bool)
+        background[ab:ab + al] = ~inside[ab:ab + al]
+        keep_slots = np.unique(full["slot_map"][~background])
+        assert part["n"] == len(keep_slots) == full["n"] - int(background.sum())
+        np.testing.assert_array_equal(part["stored"], full["stored"][keep_slots])
+        np.testing.assert_array_equal(part["exact"], full["exact"][keep_slots])
+        np.testing.assert_array_equal(part["pos"], full["pos"][keep_slots])
+        assert np.all(part["slot_map"][background] == -1)
+        remap = np.full(full["n"], -1)
+        remap[keep_slots] = np.arange(len(keep_slots))
+        np.testing.assert_array_equal(part["slot_map"][~background], remap[full["slot_map"][~background]])
+
+
+def pin_segments_hand(orc):
+    """Hand-worked confidence filter and Eq. 3 time-to-index map."""
+    g = _golden("eq3_segments.json")
+    r = orc.segments_to_spans(g["t_start"], g["t_end"], g["confidence"], g["text_len"], g["tau_total"],
+                              g["La"], g["audio_begin"], g["threshold"])
+    np.testing.assert_array_equal(r["start"], g["expected_start"])
+    np.testing.assert_array_equal(r["end"], g["expected_end"])
+    np.testing.assert_array_equal(r["groups"], g["expected_groups"])
+    np.testing.assert_array_equal(r["seg_index"], g["expected_seg_index"])
+
+
+def pin_segments_properties(orc):
+    """On random ASR output the spans are sorted, disjoint, inside the audio region; exactly the
+    segments above the threshold are kept, with their text lengths; where segments neither
+    overlap nor leave the audio, an interval's length is the number of token boundaries
+    k / L_a * tau_total (k integer) its times enclose, counted by brute force."""
+    rng = np.random.default_rng(6)
+    for trial in range(30):
+        La = int(rng.integers(1, 400))
+        tau = float(rng.uniform(1.0, 100.0))
+        n = int(rng.integers(0, 12))
+        cuts = np.sort(rng.uniform(0.0, tau, 2 * n))
+        ts, te = cuts[0::2], cuts[1::2]
+        conf = rng.uniform(0.0, 1.0, n)
+        tl = rng.integers(1, 6, n)
+        ab = int(rng.integers(0, 50))
+        r = orc.segments_to_spans(ts, te, conf, tl, tau, La, ab, 0.3)
+        kept = np.nonzero(conf > 0.3)[0]
+        np.testing.assert_array_equal(r["seg_index"], kept)
+        np.testing.assert_array_equal(r["groups"], tl[kept])
+        st, en = r["start"], r["end"]
+        assert np.all(st >= ab) and np.all(en <= ab + La) and np.all(en >= st)
+        assert np.all(st[1:] >= en[:-1])
+        for k, i in enumerate(kept):
+            # Token k' starts at time k' * tau / La; idx(t) = number of token starts in (0, t].
+            bounds = np.arange(1, La + 1) * (tau / La)
+            lo = int(np.sum(bounds <= ts[i] * (1 + 1e-12)))
+            hi = int(np.sum(bounds <= te[i] * (1 + 1e-12)))
+            near = lambda t: np.min(np.abs(bounds - t)) < 1e-9 * tau
+            if not (near(ts[i]) or near(te[i])):
+                assert st[k] - ab == lo and en[k] - ab == hi, (trial, i, st[k] - ab, lo, en[k] - ab, hi)
+    # Overlapping or unsorted input: overlaps are clipped, unsorted input is rejected.
+    r = orc.segments_to_spans([0.0, 0.5], [1.0, 2.0], [1.0, 1.0], [1, 1], 2.0, 20)
+    np.testing.assert_array_equal(r["start"], [0, 10]) and np.testing.assert_array_equal(r["end"], [10, 20])
+    for args in (([1.0, 0.5], [2.0, 2.0], [1.0, 1.0], [1, 1], 2.0, 20),   # unsorted
+                 ([0.0], [1.0], [1.0], [0], 2.0, 20),                       # no text tokens
+                 ([0.0], [1.0], [1.0], [1], 0.0, 20),                       # zero duration
+                 ([1.0], [0.5], [1.0], [1], 2.0, 20)):                      # ends before it starts
+        try:
+            orc.segments_to_spans(*args)
+        except O.OracleError:
+            continue
+        raise AssertionError(f"accepted {args}")
+
+
 def pin_stage1_errors(orc):
     """Malformed semantic sets are rejected; the output must fit the capacity."""
     x = np.zeros((10, 4))

@@ -52,6 +52,18 @@ MUTATIONS = [
      "for (int32_t j = 0; j < T - 1; ++j)\n        keep[j] = 1;"),
     ("score not moved with its row", "score[w] = score[j];", "(void)0;"),
     ("position not moved with its row", "pos[w] = pos[j];", "(void)0;"),
+    ("confidence filter keeps the threshold itself", "if (!(confidence[i] > threshold))",
+     "if (!(confidence[i] >= threshold))"),
+    ("Eq. 3 rounds instead of flooring", "double fs = floor((double)La * (t_start[i] / tau_total));",
+     "double fs = round((double)La * (t_start[i] / tau_total));"),
+    ("Eq. 3 end index rounded up", "double fe = floor((double)La * (t_end[i] / tau_total));",
+     "double fe = ceil((double)La * (t_end[i] / tau_total));"),
+    ("overlapping segments not clipped", "        if (s < prev_end)\n            s = prev_end;\n", ""),
+    ("segment text length not carried", "span_groups[kept] = text_len[i];", "span_groups[kept] = 1;"),
+    ("Partial keeps the background", "} else if (!keep_background && t >= audio_begin && t < audio_begin + audio_len) {",
+     "} else if (0) {"),
+    ("Partial drops the text too", "} else if (!keep_background && t >= audio_begin && t < audio_begin + audio_len) {",
+     "} else if (!keep_background) {"),
     ("margin against the wrong runner-up", "*margin = c[N - 1].score - c[N].score;",
      "*margin = c[N - 1].score - c[N + 1 < nc ? N + 1 : N].score;"),
 ]
