@@ -8,6 +8,11 @@ The reported value is decode steps per second of the whole job (each decode step
 sequence of the batch by one token through all layers), stage 1 and evictions included.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload stress] [--impl voxzip|reference]
+  python bench.py --part embed [--steps K] [--warmup W]
+
+`--part embed` measures stage 1 where the paper runs it instead: ASR segments of 4 x 60 min of
+audio to spans (Eq. 3, on the host) and the fusion of the prompt embeddings (d_model 2048) with the
+embedded transcriptions as anchors; one step fuses the four sequences once.
 
 Under torchrun each rank runs its own replica of the workload on its own GPU (the units of the
 path are independent, so there is no data-path collective); the time is the max over ranks.
@@ -47,6 +52,8 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-units", type=int, default=0, help="units in the oracle sample (0: one per core)")
+    p.add_argument("--part", choices=["path", "embed"], default="path",
+                   help="path: the KV-compression path (default); embed: embedding-level stage 1")
     return p.parse_args()
 
 
@@ -512,9 +519,203 @@ def reference_arm(args, rank, world):
             "e2e": {"value": round(value, 4), "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+# ----------------------------------------------------------------------------- embedding-level stage 1
+
+EMBED_METRIC = "stage-1 embedding fusion (Sec. 3.2.1, Eq. 3-5): sequences/s, 4 x 60 min audio, d_model 2048"
+
+
+class EmbedRunner:
+    """Resident inputs of embedding-level stage 1: prompt embeddings, spans from the ASR
+    segments (the library's Eq. 3 helper), and the kept segments' text embeddings."""
+
+    def __init__(self, w, device):
+        from paper_2608_08569_gb300 import EmbedDesc, voxzip_segments_to_spans
+        from paper_2608_08569_gb300 import workloads as W
+        self.w, self.dev = w, device
+        self.segs = W.make_segments(w)
+        self.e_in = W.make_embeddings(w, device)
+        self.text_all = W.make_text_embeddings(w, self.segs, device)
+        self.spans_host()
+        off, st, en, gr = self.spans
+        i32 = lambda x: torch.as_tensor(np.asarray(x), dtype=torch.int32, device=device)
+        self.args = [i32(w.in_len), i32([w.audio_begin] * w.batch), i32(w.audio_len), i32(off), i32(st), i32(en),
+                     i32(gr)]
+        rows = []
+        for b, s in enumerate(self.segs):
+            first = np.concatenate([[0], np.cumsum(s.text_len)])
+            sel = [np.arange(first[i], first[i + 1]) for i in self.seg_index[b]]
+            rows.append(np.concatenate(sel) if sel else np.zeros(0, np.int64))
+        self.e_text = torch.zeros(w.batch, max(1, max(len(r) for r in rows)), w.d_model, dtype=w.dtype, device=device)
+        for b, r in enumerate(rows):
+            if len(r):
+                self.e_text[b, :len(r)] = self.text_all[b, torch.as_tensor(r, device=device)]
+        self.desc = EmbedDesc(w.batch, w.d_model, w.capacity, w.dtype)
+        self.out = torch.empty(w.batch, w.capacity, w.d_model, dtype=w.dtype, device=device)
+        self.pos = torch.empty(w.batch, w.capacity, dtype=torch.int32, device=device)
+        self.len = torch.empty(w.batch, dtype=torch.int32, device=device)
+
+    def spans_host(self):
+        """The semantic set of every sequence from its ASR segments (host, Eq. 3)."""
+        from paper_2608_08569_gb300 import voxzip_segments_to_spans
+        w = self.w
+        off, st, en, gr, self.seg_index = [0], [], [], [], []
+        for b, s in enumerate(self.segs):
+            r = voxzip_segments_to_spans(s.t_start, s.t_end, s.confidence, s.text_len, s.tau_total, w.audio_len[b],
+                                         w.audio_begin)
+            st += list(r["start"]); en += list(r["end"]); gr += list(r["groups"])
+            self.seg_index.append(r["seg_index"])
+            off.append(len(st))
+        self.spans = (off, st, en, gr)
+
+    def step(self):
+        from paper_2608_08569_gb300 import voxzip_embed_fuse
+        voxzip_embed_fuse(self.desc, self.e_in, *self.args, self.out, self.pos, self.len, e_text=self.e_text)
+
+    def alg_bytes(self):
+        """Embedding rows read (prompt, and one text row per emitted group), fused rows written,
+        and the per-row integers (position; source range and anchor row written and read)."""
+        w, e = self.w, (2 if self.w.dtype == torch.bfloat16 else 4)
+        off, st, en, gr = self.spans
+        groups = sum(min(g, b - a) for a, b, g in zip(st, en, gr))
+        n_out = int(self.len.sum())
+        return (sum(w.in_len) + groups + n_out) * w.d_model * e + n_out * 28 + len(st) * 12
+
+
+def embed_arm(args, rank, world, local):
+    from paper_2608_08569_gb300 import voxzip_get_status
+    from paper_2608_08569_gb300 import workloads as W
+    w = W.EMBED_CONFIGS["embed_stress"]
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    r = EmbedRunner(w, dev)
+    for _ in range(args.warmup):
+        r.step()
+    torch.cuda.synchronize()
+    if voxzip_get_status() != 0:
+        raise RuntimeError("device status word set by embedding-level stage 1")
+    barrier(world)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(local) as clk:
+        torch.cuda.synchronize()
+        barrier(world)
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        e0.record()
+        for a, b in evs:
+            a.record()
+            r.step()
+            b.record()
+        e1.record()
+        torch.cuda.synchronize()
+        barrier(world)
+    ms = e0.elapsed_time(e1)
+    ms_max = max_over_ranks(ms, world)
+    value = world * args.steps * w.batch / (ms_max / 1000.0)
+    launch_ms = sum(a.elapsed_time(b) for a, b in evs) / args.steps
+    alg = r.alg_bytes()
+    peak, peak_kind = peaks()
+    achieved = alg / (launch_ms / 1000.0) / 1e9
+    roofline = {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "traffic": None,
+                "kernel": "embedding stage 1 (span_scan + slot_map + fuse_wide_kernel, timed together)",
+                "peak_source": f"{peak_kind} hbm_gbs", "avg_call_us": round(launch_ms * 1000.0, 2),
+                "alg_bytes_per_call": int(alg)}
+    e2e = None if args.no_e2e else embed_e2e(r, args)
+    clocks = clk.summary()
+    result = {
+        "metric": EMBED_METRIC, "value": round(value, 2), "unit": "sequences/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 3),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "bf16" if w.dtype == torch.bfloat16 else "f32",
+        "data": "synthetic (seeded; N(0,1) embeddings, ASR-like timed segments at 12.5 audio tokens/s)",
+        "config": {"workload": f"{w.name}: {w.description}", "batch": w.batch, "d_model": w.d_model,
+                   "prompt_tokens": list(sorted(set(w.in_len))), "spans": len(r.spans[1]),
+                   "output_rows": int(r.len.sum()), "parallelism": f"replicas x{world}",
+                   "l2": "inputs larger than L2 (0.75 GB of embeddings read per step, L2 is 129 MB)"},
+        "roofline": roofline, "gpu_launches": 3 * args.steps, "clocks": clocks, "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        result["cpu_baseline"] = embed_cpu_sample(r)
+    return result
+
+
+def embed_e2e(r, args):
+    """The same with every step's embeddings and text rows copied from pinned host memory, the
+    spans recomputed from the ASR segments on the host (Eq. 3) and copied, and the fused rows
+    copied back."""
+    nbytes = lambda t: t.numel() * t.element_size()
+    h_in = torch.empty(r.e_in.shape, dtype=r.e_in.dtype, pin_memory=True)
+    h_in.copy_(r.e_in)
+    h_text = torch.empty(r.e_text.shape, dtype=r.e_text.dtype, pin_memory=True)
+    h_text.copy_(r.e_text)
+    h_out = torch.empty(r.out.shape, dtype=r.out.dtype, pin_memory=True)
+    span_bytes = [0]
+
+    def step():
+        r.spans_host()
+        off, st, en, gr = r.spans
+        hs = [torch.as_tensor(np.asarray(x), dtype=torch.int32).pin_memory() for x in (off, st, en, gr)]
+        for src, dst in zip(hs, r.args[3:]):
+            dst.copy_(src, non_blocking=True)
+        span_bytes[0] = sum(nbytes(t) for t in hs)
+        r.e_in.copy_(h_in, non_blocking=True)
+        r.e_text.copy_(h_text, non_blocking=True)
+        r.step()
+        h_out.copy_(r.out, non_blocking=True)
+
+    step()
+    torch.cuda.synchronize()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for _ in range(args.steps):
+        step()
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    return {"value": round(args.steps * r.w.batch / (ms / 1000.0), 2), "unit": "sequences/s",
+            "h2d_bytes_per_step": nbytes(h_in) + nbytes(h_text) + span_bytes[0],
+            "d2h_bytes_per_step": nbytes(h_out), "ms_per_step": round(ms / args.steps, 3)}
+
+
+def embed_cpu_sample(r, cols=16):
+    """The oracle's stage 1 on `cols` of the d_model columns of every sequence (stage 1 acts on
+    each column alone), one sequence per thread; scaled to whole sequences per second."""
+    import oracle
+    w = r.w
+    oracle.build()
+    off, st, en, gr = r.spans
+    sel = torch.arange(0, w.d_model, w.d_model // cols, device=r.e_in.device)[:cols]
+    xs = [r.e_in[b, :w.in_len[b]][:, sel].double().cpu().numpy() for b in range(w.batch)]
+    ts = [r.e_text[b][:, sel].double().cpu().numpy() for b in range(w.batch)]
+
+    def one(b):
+        s0, s1 = off[b], off[b + 1]
+        oracle.stage1(xs[b], w.in_len[b], w.audio_begin, w.audio_len[b], st[s0:s1], en[s0:s1], gr[s0:s1],
+                      anchor=ts[b], cache_is_bf16=True, capacity=w.capacity)
+
+    threads = min(cores(), w.batch)
+    t0 = time.perf_counter()
+    with cf.ThreadPoolExecutor(threads) as ex:
+        list(ex.map(one, range(w.batch)))
+    sec = time.perf_counter() - t0
+    per_seq = sec / w.batch * threads * (w.d_model / cols)
+    return {"value": round(threads / per_seq, 4), "unit": "sequences/s", "cores": threads, "kind": "oracle",
+            "sample": f"{cols} of {w.d_model} columns of each of the {w.batch} sequences (all rows), one thread "
+                      f"per sequence; scaled by d_model / {cols}"}
+
+
 def main():
     args = parse_args()
     rank, world, local = dist_setup()
+    if args.part == "embed" and args.impl != "reference":
+        res = embed_arm(args, rank, world, local)
+        if rank == 0:
+            print(json.dumps(res), flush=True)
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+        return
     if args.impl == "reference":
         res = reference_arm(args, rank, world)
     else:

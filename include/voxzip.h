@@ -8,7 +8,9 @@
  *           (Eq. 6), updated by every decode step (Eq. 1-2), and evicts down to a budget
  *           by keeping T sinks, a recent window of M tokens and the top-N scored history
  *           (Eq. 7-9).
- * The library exports one call per step: voxzip_anchor_fuse, voxzip_decode_step, voxzip_evict.
+ * The library exports one call per step: voxzip_anchor_fuse, voxzip_decode_step, voxzip_evict;
+ * and, for stage 1 where the paper runs it (on input embeddings, from ASR segments),
+ * voxzip_segments_to_spans (host) and voxzip_embed_fuse.
  *
  * Conventions shared by every entry point
  *   - A "unit" is one (sequence b, layer l, kv-head h). All state is per unit and units are
@@ -141,6 +143,80 @@ voxzip_status voxzip_anchor_fuse_noalloc(const voxzip_cache_desc *desc, const vo
                                          int32_t anchor_stride, void *k_cache, void *v_cache,
                                          float *score, int32_t *pos, int32_t *len,
                                          int32_t *slot_map, voxzip_stream_t stream);
+
+/*
+ * The semantic set of one sequence from ASR output (Sec. 3.2.1): the confidence filter and the
+ * time-to-index map of Eq. 3. HOST function: every pointer is host memory; no CUDA call, no GPU.
+ *
+ * Segment i (times in seconds, sorted by t_start) is kept when confidence[i] > threshold (the
+ * paper keeps segments above 0.3). Its interval of audio tokens is
+ *     [floor(audio_len * (t_start / tau_total)), floor(audio_len * (t_end / tau_total)))   (Eq. 3)
+ * evaluated in double in that order and clamped to [0, audio_len]. A kept segment that would
+ * start before the previous kept one ends starts where that one ends (an empty interval if
+ * nothing is left: it yields no row, but its text rows still count for the anchor offsets).
+ *
+ *   t_start, t_end, confidence  [n] double; text_len [n] int32 >= 1 (L_t, the segment's tokens)
+ *   tau_total      duration of the audio, seconds, finite and > 0
+ *   audio_len      L_a, audio tokens; audio_begin = prompt index of the first one
+ *   span_start, span_end, span_groups, seg_index   outputs, room for n entries each: the kept
+ *                  segments in order as prompt-index spans, their L_t, and their input index
+ *   num_spans      output: number of kept segments
+ * The outputs feed voxzip_anchor_fuse / voxzip_embed_fuse (span_groups = n_groups; the anchor
+ * rows are the embedded texts of the kept segments, concatenated in this order).
+ * Errors: VOXZIP_EINVAL for n < 0, a NULL pointer (with n > 0), unsorted segments,
+ * t_end < t_start (or NaN), text_len < 1, a bad tau_total, audio_len or audio_begin < 0.
+ */
+voxzip_status voxzip_segments_to_spans(int32_t n, const double *t_start, const double *t_end,
+                                       const double *confidence, const int32_t *text_len,
+                                       double tau_total, int32_t audio_len, int32_t audio_begin,
+                                       double threshold, int32_t *span_start, int32_t *span_end,
+                                       int32_t *span_groups, int32_t *seg_index,
+                                       int32_t *num_spans);
+
+typedef struct {
+    int32_t batch;    /* B, sequences */
+    int32_t d_model;  /* d, hidden size; rows are whole 16-byte vectors (multiple of 8 bf16 or
+                         4 fp32 elements) */
+    int32_t capacity; /* C, output rows per sequence */
+    int32_t dtype;    /* voxzip_dtype of e_in, e_text and e_out */
+} voxzip_embed_desc;
+
+/*
+ * Stage 1 at the embedding level, the setting the paper evaluates (Sec. 3.2.1): the audio
+ * embeddings E_A of each sequence are fused under its semantic set before the LLM runs. Group j
+ * of a span (Eq. 4 grouping, as in voxzip_anchor_fuse) becomes mean(E_A rows of the group) +
+ * e_t,j, the j-th embedded text token of the span's transcription (the semantic anchor);
+ * background audio and every token outside the audio region are copied (Eq. 5).
+ *
+ * keep_background = 0 gives the stage-1 ablation's T+A (Partial) configuration: audio that no
+ * span covers is dropped (slot_map -1), text outside the audio region is still copied.
+ *
+ *   e_in        [B][stride][d] prompt embeddings; rows [0, in_len[b]) are read; the audio
+ *               region is [audio_begin[b], audio_begin[b] + audio_len[b])
+ *   in_len, audio_begin, audio_len, span_off, span_start, span_end, span_groups
+ *               device int32, exactly as for voxzip_anchor_fuse
+ *   e_text      NULL (no anchor term) or [B][text_stride][d]: sequence b's embedded texts,
+ *               concatenated in span order; group j of span i adds row
+ *               (sum of span_groups over b's spans before i) + j
+ *   e_out       [B][capacity][d] output rows; pos [B][capacity] int32: first prompt token of each
+ *               output row; len [B] int32: output rows per sequence
+ *   slot_map    NULL or [B][stride] int32: output row of every prompt token, -1 if dropped
+ *   workspace   device scratch of voxzip_embed_fuse_workspace_size() bytes, 256-byte aligned
+ * All tensor pointers are device memory, 16-byte aligned. Device errors: VOXZIP_DEV_BAD_SPANS or
+ * VOXZIP_DEV_CAPACITY skip the sequence (len = 0).
+ */
+voxzip_status voxzip_embed_fuse(const voxzip_embed_desc *desc, const void *e_in, int32_t stride,
+                                const int32_t *in_len, const int32_t *audio_begin,
+                                const int32_t *audio_len, const int32_t *span_off,
+                                int32_t num_spans, const int32_t *span_start,
+                                const int32_t *span_end, const int32_t *span_groups,
+                                const void *e_text, int32_t text_stride, int32_t keep_background,
+                                void *e_out, int32_t *pos, int32_t *len, int32_t *slot_map,
+                                void *workspace, size_t workspace_bytes, voxzip_stream_t stream);
+
+/* Bytes of workspace voxzip_embed_fuse needs (0 if the arguments are invalid). */
+size_t voxzip_embed_fuse_workspace_size(const voxzip_embed_desc *desc, int32_t stride,
+                                        int32_t num_spans);
 
 /*
  * One decode step for layers [layer_begin, layer_begin + layer_count) of every sequence:

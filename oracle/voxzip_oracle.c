@@ -202,7 +202,8 @@ int vzo_stage1(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t n
  *   span_groups            L_t of the segment
  *   seg_index              which input segment it came from
  *   n_spans                how many were kept
- * Returns VZO_EINVAL for unsorted segments, t_end < t_start, L_t < 1 or tau_total <= 0.
+ * Returns VZO_EINVAL for unsorted segments, t_end < t_start, L_t < 1, or a duration that is not
+ * finite and positive (Eq. 3 divides by it).
  */
 int vzo_segments_to_spans(int32_t n_seg, const double *t_start, const double *t_end,
                           const double *confidence, const int32_t *text_len, double tau_total,
@@ -210,7 +211,7 @@ int vzo_segments_to_spans(int32_t n_seg, const double *t_start, const double *t_
                           int32_t *span_end, int32_t *span_groups, int32_t *seg_index,
                           int32_t *n_spans)
 {
-    if (n_seg < 0 || !(tau_total > 0.0) || La < 0 || audio_begin < 0)
+    if (n_seg < 0 || !(tau_total > 0.0) || isinf(tau_total) || La < 0 || audio_begin < 0)
         return VZO_EINVAL;
     for (int32_t i = 0; i < n_seg; ++i) {
         if (!(t_end[i] >= t_start[i]) || text_len[i] < 1 || (i > 0 && t_start[i] < t_start[i - 1]))

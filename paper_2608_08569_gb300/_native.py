@@ -54,13 +54,32 @@ class CacheDesc:
                      _DTYPES[self.dtype])
 
 
+class _EmbedDesc(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("d_model", ctypes.c_int32), ("capacity", ctypes.c_int32),
+                ("dtype", ctypes.c_int32)]
+
+
+@dataclass(frozen=True)
+class EmbedDesc:
+    """Shape of embedding-level stage 1: B sequences, output rows of d_model elements, C rows each."""
+    batch: int
+    d_model: int
+    capacity: int
+    dtype: torch.dtype = torch.bfloat16
+
+    def c_struct(self) -> _EmbedDesc:
+        return _EmbedDesc(self.batch, self.d_model, self.capacity, _DTYPES[self.dtype])
+
+
 _lock = threading.Lock()
 _lib = None
 _vp = ctypes.c_void_p
 _i32 = ctypes.c_int32
 _f32 = ctypes.c_float
 _sz = ctypes.c_size_t
+_f64 = ctypes.c_double
 _DP = ctypes.POINTER(_Desc)
+_EP = ctypes.POINTER(_EmbedDesc)
 
 
 def lib() -> ctypes.CDLL:
@@ -82,10 +101,17 @@ def lib() -> ctypes.CDLL:
                                              _f32, _f32, _i32, _vp, _vp]
             L.voxzip_evict.argtypes = [_DP, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _f32, _vp]
             L.voxzip_get_status.argtypes = [ctypes.POINTER(ctypes.c_uint32), _vp]
+            L.voxzip_segments_to_spans.argtypes = [_i32, _vp, _vp, _vp, _vp, _f64, _i32, _i32, _f64, _vp, _vp, _vp,
+                                                   _vp, _vp]
+            L.voxzip_embed_fuse.argtypes = [_EP, _vp, _i32, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _i32,
+                                            _i32, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+            L.voxzip_embed_fuse_workspace_size.argtypes = [_EP, _i32, _i32]
+            L.voxzip_embed_fuse_workspace_size.restype = _sz
             L.voxzip_status_string.argtypes = [_i32]
             L.voxzip_status_string.restype = ctypes.c_char_p
             L.voxzip_version.restype = _i32
-            for f in (L.voxzip_anchor_fuse, L.voxzip_decode_step, L.voxzip_evict, L.voxzip_get_status):
+            for f in (L.voxzip_anchor_fuse, L.voxzip_decode_step, L.voxzip_evict, L.voxzip_get_status,
+                      L.voxzip_segments_to_spans, L.voxzip_embed_fuse):
                 f.restype = _i32
             _lib = L
     return _lib
@@ -176,6 +202,71 @@ def voxzip_anchor_fuse(desc: CacheDesc, k_prefill, v_prefill, in_len, audio_begi
         _ptr(audio_len), _ptr(span_off), int(num_spans), _ptr(span_start), _ptr(span_end), _ptr(span_groups),
         _ptr(anchor_k), _ptr(anchor_v), int(anchor_stride), _ptr(k_cache), _ptr(v_cache), _ptr(score),
         _ptr(pos), _ptr(len_), _ptr(slot_map), _ptr(workspace), int(workspace.numel()), _stream(stream)))
+
+
+def voxzip_segments_to_spans(t_start, t_end, confidence, text_len, tau_total: float, audio_len: int,
+                             audio_begin: int = 0, threshold: float = 0.3) -> dict:
+    """ASR segments -> token-index spans (host): the confidence filter and Eq. 3. Returns
+    dict(start, end, groups, seg_index) of int32 numpy arrays, one entry per kept segment."""
+    import numpy as np
+    ts = np.ascontiguousarray(t_start, dtype=np.float64)
+    te = np.ascontiguousarray(t_end, dtype=np.float64)
+    cf = np.ascontiguousarray(confidence, dtype=np.float64)
+    tl = np.ascontiguousarray(text_len, dtype=np.int32)
+    n = len(ts)
+    if not (len(te) == n and len(cf) == n and len(tl) == n):
+        raise ValueError("t_start, t_end, confidence and text_len must have the same length")
+    outs = [np.zeros(max(n, 1), np.int32) for _ in range(4)]
+    k = ctypes.c_int32(0)
+    p = lambda a: a.ctypes.data_as(ctypes.c_void_p)
+    _check("voxzip_segments_to_spans", lib().voxzip_segments_to_spans(
+        n, p(ts), p(te), p(cf), p(tl), float(tau_total), int(audio_len), int(audio_begin), float(threshold),
+        *[p(a) for a in outs], ctypes.byref(k)))
+    m = k.value
+    return dict(start=outs[0][:m], end=outs[1][:m], groups=outs[2][:m], seg_index=outs[3][:m])
+
+
+def voxzip_embed_fuse_workspace_size(desc: EmbedDesc, stride: int, num_spans: int) -> int:
+    d = desc.c_struct()
+    return int(lib().voxzip_embed_fuse_workspace_size(ctypes.byref(d), int(stride), int(num_spans)))
+
+
+def voxzip_embed_fuse(desc: EmbedDesc, e_in, in_len, audio_begin, audio_len, span_off, span_start, span_end,
+                      span_groups, e_out, pos, len_, *, e_text=None, keep_background: bool = True, slot_map=None,
+                      workspace=None, stream=None) -> None:
+    """Stage 1 at the embedding level (Sec. 3.2.1): fuse each sequence's audio embeddings under its
+    semantic set, adding the embedded transcription as anchors; keep_background=False is the
+    "Partial" configuration (uncovered audio dropped)."""
+    B, D, C = desc.batch, desc.d_model, desc.capacity
+    if e_in.dim() != 3:
+        raise ValueError("e_in must be [B][stride][d_model]")
+    stride = e_in.shape[1]
+    _need(e_in, "e_in", desc.dtype, (B, stride, D))
+    for name, t in (("in_len", in_len), ("audio_begin", audio_begin), ("audio_len", audio_len)):
+        _need(t, name, torch.int32, (B,))
+    _need(span_off, "span_off", torch.int32, (B + 1,))
+    num_spans = span_start.numel()
+    for name, t in (("span_start", span_start), ("span_end", span_end), ("span_groups", span_groups)):
+        _need(t, name, torch.int32, (num_spans,))
+    _need(e_out, "e_out", desc.dtype, (B, C, D))
+    _need(pos, "pos", torch.int32, (B, C))
+    _need(len_, "len", torch.int32, (B,))
+    if slot_map is not None:
+        _need(slot_map, "slot_map", torch.int32, (B, stride))
+    text_stride = 0
+    if e_text is not None:
+        text_stride = e_text.shape[1]
+        _need(e_text, "e_text", desc.dtype, (B, text_stride, D))
+    need = voxzip_embed_fuse_workspace_size(desc, stride, num_spans)
+    if workspace is None:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=e_out.device)
+    _need(workspace, "workspace", torch.uint8)
+    d = desc.c_struct()
+    _check("voxzip_embed_fuse", lib().voxzip_embed_fuse(
+        ctypes.byref(d), _ptr(e_in), int(stride), _ptr(in_len), _ptr(audio_begin), _ptr(audio_len), _ptr(span_off),
+        int(num_spans), _ptr(span_start), _ptr(span_end), _ptr(span_groups), _ptr(e_text), int(text_stride),
+        int(bool(keep_background)), _ptr(e_out), _ptr(pos), _ptr(len_), _ptr(slot_map), _ptr(workspace),
+        int(workspace.numel()), _stream(stream)))
 
 
 def voxzip_anchor_fuse_noalloc(desc: CacheDesc, k_prefill, v_prefill, in_len, audio_begin, audio_len, span_off,

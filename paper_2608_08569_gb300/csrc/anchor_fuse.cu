@@ -1,18 +1,23 @@
-// Stage 1 of VoxZip (Sec. 3.2.1): semantic-anchored fusion of the prefilled K/V cache.
+// Stage 1 of VoxZip (Sec. 3.2.1): semantic-anchored fusion of the prefilled K/V cache, or of the
+// input embeddings (the paper's own setting).
 //
-// Three kernels, all launched on the caller's stream:
+// Kernels, all launched on the caller's stream:
 //   span_scan   one CTA per sequence: validates the semantic set (sorted, non-overlapping spans
 //               inside the audio region) and scans, per span, the slot shift
-//               delta = min(n_groups, l) - l and the anchor-row offset (prefix of n_groups);
-//   slot_map    one thread per prefill token: the output slot of the token (Eq. 4 grouping with
+//               delta = min(n_groups, l) - l, the anchor-row offset (prefix of n_groups) and the
+//               background tokens before the span (dropped in the "Partial" configuration);
+//   slot_map    one thread per prompt token: the output slot of the token (Eq. 4 grouping with
 //               group j = [floor(j*l/g), floor((j+1)*l/g)), Eq. 5 chronological order); the first
-//               token of each slot records the slot's source range start and anchor row;
-//   fuse_rows   one warp-slice per output slot of every (layer, kv-head) unit: the fp32 mean of
-//               the slot's source rows (a copy when the range has one row) plus the anchor row,
-//               rounded once to the cache dtype; K and V in the same pass; pos and score = 0.
-// Output slots tile the prompt into contiguous ranges in order, so a slot is fully described by
-// the first token of its range; the range ends where the next slot's begins.
+//               token of each slot records the slot's source range and anchor row;
+//   fuse_rows   K/V level, head_dim 64 or 128: one warp-slice per output slot of every (layer,
+//               kv-head) unit: the fp32 mean of the slot's source rows (a copy when the range has
+//               one row) plus the anchor row, rounded once to the cache dtype; K and V in the same
+//               pass; pos and score = 0;
+//   fuse_wide   embedding level, any width that is a whole number of 16-byte vectors: one warp per
+//               output row of a sequence, the same arithmetic.
+// Output slots cover the kept tokens of the prompt in order, each a contiguous source range.
 #include "common.cuh"
+#include "embed.cuh"
 
 namespace voxzip {
 namespace {
@@ -24,9 +29,12 @@ constexpr int kSlotsPerWarp = 8;
 
 struct FuseWorkspace {
     int32_t *seq_len;        // [B] stage-1 length, -1 when the sequence is skipped
+    int32_t *bg_total;       // [B] background (uncovered audio) tokens of the sequence
     int32_t *delta_prefix;   // [num_spans] exclusive prefix of (g - l) within the sequence
     int32_t *anchor_prefix;  // [num_spans] exclusive prefix of n_groups within the sequence
-    int32_t *slot_src;       // [B][stride + 1] first prefill token of each slot, then in_len
+    int32_t *bg_prefix;      // [num_spans] background tokens before the span's start
+    int32_t *slot_src;       // [B][stride] first prompt token of each slot
+    int32_t *slot_end;       // [B][stride] one past the last prompt token of each slot
     int32_t *slot_anchor;    // [B][stride] anchor row of each slot, -1 for copied rows
 };
 
@@ -41,15 +49,21 @@ __host__ __device__ inline size_t carve(const voxzip_cache_desc &d, int32_t stri
         return reinterpret_cast<int32_t *>(p);
     };
     int32_t *a = take(sizeof(int32_t) * (size_t)d.batch);
+    int32_t *a2 = take(sizeof(int32_t) * (size_t)d.batch);
     int32_t *b = take(sizeof(int32_t) * (size_t)num_spans);
     int32_t *c = take(sizeof(int32_t) * (size_t)num_spans);
-    int32_t *e = take(sizeof(int32_t) * (size_t)d.batch * ((size_t)stride + 1));
+    int32_t *c2 = take(sizeof(int32_t) * (size_t)num_spans);
+    int32_t *e = take(sizeof(int32_t) * (size_t)d.batch * (size_t)stride);
+    int32_t *e2 = take(sizeof(int32_t) * (size_t)d.batch * (size_t)stride);
     int32_t *f = take(sizeof(int32_t) * (size_t)d.batch * (size_t)stride);
     if (ws) {
         ws->seq_len = a;
+        ws->bg_total = a2;
         ws->delta_prefix = b;
         ws->anchor_prefix = c;
+        ws->bg_prefix = c2;
         ws->slot_src = e;
+        ws->slot_end = e2;
         ws->slot_anchor = f;
     }
     return off;
@@ -85,7 +99,7 @@ __device__ int block_excl_scan(int v, int *total) {
 
 __global__ void __launch_bounds__(kScanThreads)
 span_scan_kernel(int32_t B, int32_t stride, int32_t capacity, int32_t num_spans, int32_t anchor_stride,
-                 bool has_anchor, const int32_t *__restrict__ in_len, const int32_t *__restrict__ audio_begin,
+                 bool has_anchor, bool keep_bg, const int32_t *__restrict__ in_len, const int32_t *__restrict__ audio_begin,
                  const int32_t *__restrict__ audio_len, const int32_t *__restrict__ span_off,
                  const int32_t *__restrict__ span_start, const int32_t *__restrict__ span_end,
                  const int32_t *__restrict__ span_groups, FuseWorkspace ws, int32_t *status) {
@@ -104,10 +118,10 @@ span_scan_kernel(int32_t B, int32_t stride, int32_t capacity, int32_t num_spans,
         }
         return;
     }
-    int carry_delta = 0, carry_groups = 0;
+    int carry_delta = 0, carry_groups = 0, carry_gap = 0;
     for (int base = s0; base < s1; base += blockDim.x) {
         const int i = base + threadIdx.x;
-        int delta = 0, groups = 0;
+        int delta = 0, groups = 0, gap = 0;
         if (i < s1) {
             const int32_t st = span_start[i], en = span_end[i], ng = span_groups[i];
             const int32_t prev_end = i > s0 ? span_end[i - 1] : ab;
@@ -115,20 +129,27 @@ span_scan_kernel(int32_t B, int32_t stride, int32_t capacity, int32_t num_spans,
             const int32_t l = en - st;
             delta = (ng < l ? ng : l) - l;
             groups = ng;
+            gap = st - prev_end;  // background audio between the previous span (or the audio start) and this one
         }
-        int tot_d, tot_g;
+        int tot_d, tot_g, tot_b;
         const int ex_d = block_excl_scan(delta, &tot_d);
         const int ex_g = block_excl_scan(groups, &tot_g);
+        const int ex_b = block_excl_scan(gap, &tot_b);
         if (i < s1) {
             ws.delta_prefix[i] = carry_delta + ex_d;
             ws.anchor_prefix[i] = carry_groups + ex_g;
+            ws.bg_prefix[i] = carry_gap + ex_b + gap;
         }
         carry_delta += tot_d;
         carry_groups += tot_g;
+        carry_gap += tot_b;
     }
     __syncthreads();
     if (threadIdx.x == 0) {
-        const int64_t out_len = (int64_t)n_in + carry_delta;
+        const int32_t last_end = s1 > s0 ? span_end[s1 - 1] : ab;
+        const int32_t bg = carry_gap + (ab + al - last_end);
+        ws.bg_total[b] = bg;
+        const int64_t out_len = (int64_t)n_in + carry_delta - (keep_bg ? 0 : bg);
         if (bad || (has_anchor && carry_groups > anchor_stride)) {
             ws.seq_len[b] = -1;
             raise_status(status, VOXZIP_DEV_BAD_SPANS);
@@ -142,9 +163,11 @@ span_scan_kernel(int32_t B, int32_t stride, int32_t capacity, int32_t num_spans,
 }
 
 __global__ void __launch_bounds__(kMapThreads)
-slot_map_kernel(int32_t stride, const int32_t *__restrict__ in_len, const int32_t *__restrict__ span_off,
-                const int32_t *__restrict__ span_start, const int32_t *__restrict__ span_end,
-                const int32_t *__restrict__ span_groups, FuseWorkspace ws, int32_t *__restrict__ slot_map) {
+slot_map_kernel(int32_t stride, bool keep_bg, const int32_t *__restrict__ in_len,
+                const int32_t *__restrict__ audio_begin, const int32_t *__restrict__ audio_len,
+                const int32_t *__restrict__ span_off, const int32_t *__restrict__ span_start,
+                const int32_t *__restrict__ span_end, const int32_t *__restrict__ span_groups, FuseWorkspace ws,
+                int32_t *__restrict__ slot_map) {
     const int b = blockIdx.y;
     const int32_t t = blockIdx.x * blockDim.x + threadIdx.x;
     const int32_t out_len = ws.seq_len[b];
@@ -159,7 +182,7 @@ slot_map_kernel(int32_t stride, const int32_t *__restrict__ in_len, const int32_
         else hi = mid;
     }
     const int i = lo - 1;
-    int32_t slot, anchor = -1;
+    int32_t slot, end, anchor = -1;
     bool first;
     if (i >= s0 && t < span_end[i]) {
         const int64_t st = span_start[i], l = span_end[i] - st;
@@ -167,22 +190,30 @@ slot_map_kernel(int32_t stride, const int32_t *__restrict__ in_len, const int32_
         const int64_t g = ng < l ? ng : l;
         const int64_t r = t - st;
         const int64_t j = ((r + 1) * g - 1) / l;  // group j holds r iff floor(j*l/g) <= r < floor((j+1)*l/g)
-        slot = (int32_t)(st + ws.delta_prefix[i] + j);
+        slot = (int32_t)(st + ws.delta_prefix[i] - (keep_bg ? 0 : ws.bg_prefix[i]) + j);
         first = r == (j * l) / g;
+        end = (int32_t)(st + ((j + 1) * l) / g);
         anchor = (int32_t)(ws.anchor_prefix[i] + j);
     } else {
-        const int32_t shift = i >= s0 ? ws.delta_prefix[i] + (min(span_groups[i], span_end[i] - span_start[i]) -
-                                                             (span_end[i] - span_start[i]))
-                                      : 0;
+        const int32_t ab = audio_begin[b], ae = ab + audio_len[b];
+        if (!keep_bg && t >= ab && t < ae) {  // background audio, dropped ("Partial")
+            if (slot_map) slot_map[(int64_t)b * stride + t] = -1;
+            return;
+        }
+        int32_t shift = i >= s0 ? ws.delta_prefix[i] + (min(span_groups[i], span_end[i] - span_start[i]) -
+                                                       (span_end[i] - span_start[i]))
+                                : 0;
+        if (!keep_bg && t >= ae) shift -= ws.bg_total[b];  // a text token after the audio
         slot = t + shift;
         first = true;
+        end = t + 1;
     }
     if (slot_map) slot_map[(int64_t)b * stride + t] = slot;
     if (first) {
-        ws.slot_src[(int64_t)b * (stride + 1) + slot] = t;
+        ws.slot_src[(int64_t)b * stride + slot] = t;
+        ws.slot_end[(int64_t)b * stride + slot] = end;
         ws.slot_anchor[(int64_t)b * stride + slot] = anchor;
     }
-    if (t == n_in - 1) ws.slot_src[(int64_t)b * (stride + 1) + out_len] = n_in;
 }
 
 template <typename T, int D>
@@ -204,13 +235,14 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
     const int64_t in_base = (int64_t)u * stride * D;
     const int64_t out_base = (int64_t)u * C * D;
     const int64_t anc_base = (int64_t)u * anchor_stride * D;
-    const int32_t *src = ws.slot_src + (int64_t)b * (stride + 1);
+    const int32_t *src = ws.slot_src + (int64_t)b * stride;
+    const int32_t *send = ws.slot_end + (int64_t)b * stride;
     const int32_t *anc = ws.slot_anchor + (int64_t)b * stride;
     const int slot0 = (blockIdx.x * kFuseWarps + warp) * kSlotsPerWarp * kRowsPerWarp;
     for (int k = 0; k < kSlotsPerWarp; ++k) {
         const int s = slot0 + k * kRowsPerWarp + sub;
         if (s >= out_len) break;
-        const int32_t r0 = src[s], r1 = src[s + 1];
+        const int32_t r0 = src[s], r1 = send[s];
         float4 sk = make_float4(0.f, 0.f, 0.f, 0.f), sv = sk;
         for (int32_t r = r0; r < r1; ++r) {
             const float4 a = load4(k_prefill + in_base + (int64_t)r * D + e);
@@ -259,6 +291,124 @@ cudaError_t launch_fuse_rows(const voxzip_cache_desc &d, int32_t stride, int32_t
     return cudaGetLastError();
 }
 
+constexpr int kWideWarps = 8;
+
+// acc[e] += element e of a 16-byte vector (4 fp32 or 8 bf16 values, low address first).
+template <typename T>
+__device__ __forceinline__ void accumulate16(float *acc, uint4 x);
+template <>
+__device__ __forceinline__ void accumulate16<float>(float *acc, uint4 x) {
+    acc[0] += __uint_as_float(x.x);
+    acc[1] += __uint_as_float(x.y);
+    acc[2] += __uint_as_float(x.z);
+    acc[3] += __uint_as_float(x.w);
+}
+template <>
+__device__ __forceinline__ void accumulate16<__nv_bfloat16>(float *acc, uint4 x) {
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        acc[2 * i] += __uint_as_float(w[i] << 16);
+        acc[2 * i + 1] += __uint_as_float(w[i] & 0xffff0000u);
+    }
+}
+// The 16-byte vector of acc rounded to T (round to nearest even).
+template <typename T>
+__device__ __forceinline__ uint4 pack16(const float *acc);
+template <>
+__device__ __forceinline__ uint4 pack16<float>(const float *acc) {
+    return make_uint4(__float_as_uint(acc[0]), __float_as_uint(acc[1]), __float_as_uint(acc[2]),
+                      __float_as_uint(acc[3]));
+}
+template <>
+__device__ __forceinline__ uint4 pack16<__nv_bfloat16>(const float *acc) {
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * i]));
+        const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * i + 1]));
+        w[i] = lo | (hi << 16);
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// Embedding-level fusion: one warp per output row of sequence b; each lane owns 16-byte vectors
+// v and v + 32 of the row (two in flight per source row). The arithmetic is fuse_rows' (fp32 sum
+// in token order, IEEE division by the group size, fp32 anchor add, one rounding).
+template <typename T>
+__global__ void __launch_bounds__(kWideWarps * 32)
+fuse_wide_kernel(int32_t C, int32_t stride, int32_t D, int32_t text_stride, const T *__restrict__ e_in,
+                 const T *__restrict__ e_text, FuseWorkspace ws, T *__restrict__ e_out, int32_t *__restrict__ pos,
+                 int32_t *__restrict__ len) {
+    constexpr int kElems = 16 / sizeof(T);
+    const int b = blockIdx.y;
+    const int32_t out_len = ws.seq_len[b];
+    if (blockIdx.x == 0 && threadIdx.x == 0) len[b] = out_len < 0 ? 0 : out_len;
+    if (out_len < 0) return;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int vecs = D / kElems;
+    const T *in = e_in + (int64_t)b * stride * D;
+    const T *txt = e_text ? e_text + (int64_t)b * text_stride * D : nullptr;
+    T *out = e_out + (int64_t)b * C * D;
+    const int32_t *src = ws.slot_src + (int64_t)b * stride;
+    const int32_t *send = ws.slot_end + (int64_t)b * stride;
+    const int32_t *anc = ws.slot_anchor + (int64_t)b * stride;
+    for (int s = blockIdx.x * kWideWarps + warp; s < out_len; s += gridDim.x * kWideWarps) {
+        const int32_t r0 = src[s], r1 = send[s], a_row = anc[s];
+        const float cnt = (float)(r1 - r0);
+        for (int v0 = lane; v0 < vecs; v0 += 64) {
+            const bool two = v0 + 32 < vecs;
+            float acc[2][kElems];
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+#pragma unroll
+                for (int e = 0; e < kElems; ++e) acc[h][e] = 0.f;
+            for (int32_t r = r0; r < r1; ++r) {
+                const T *row = in + (int64_t)r * D;
+                const uint4 x0 = *reinterpret_cast<const uint4 *>(row + v0 * kElems);
+                const uint4 x1 = two ? *reinterpret_cast<const uint4 *>(row + (v0 + 32) * kElems) : x0;
+                accumulate16<T>(acc[0], x0);
+                accumulate16<T>(acc[1], x1);
+            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                if (h == 1 && !two) break;
+                const int v = v0 + 32 * h;
+                if (r1 - r0 > 1)
+#pragma unroll
+                    for (int e = 0; e < kElems; ++e) acc[h][e] = __fdiv_rn(acc[h][e], cnt);
+                if (txt != nullptr && a_row >= 0) {
+                    float t[kElems];
+#pragma unroll
+                    for (int e = 0; e < kElems; ++e) t[e] = 0.f;
+                    accumulate16<T>(t, *reinterpret_cast<const uint4 *>(txt + (int64_t)a_row * D + v * kElems));
+#pragma unroll
+                    for (int e = 0; e < kElems; ++e) acc[h][e] = __fadd_rn(acc[h][e], t[e]);
+                }
+                *reinterpret_cast<uint4 *>(out + (int64_t)s * D + v * kElems) = pack16<T>(acc[h]);
+            }
+        }
+        if (lane == 0) pos[(int64_t)b * C + s] = r0;
+    }
+}
+
+// span_scan then slot_map: the slot, source range and anchor row of every output row.
+cudaError_t launch_slot_plan(int32_t B, int32_t capacity, int32_t stride, int32_t num_spans, int32_t anchor_stride,
+                             bool has_anchor, bool keep_bg, const int32_t *in_len, const int32_t *audio_begin,
+                             const int32_t *audio_len, const int32_t *span_off, const int32_t *span_start,
+                             const int32_t *span_end, const int32_t *span_groups, const FuseWorkspace &ws,
+                             int32_t *slot_map, int32_t *status, cudaStream_t stream) {
+    span_scan_kernel<<<B, kScanThreads, 0, stream>>>(B, stride, capacity, num_spans, anchor_stride, has_anchor,
+                                                    keep_bg, in_len, audio_begin, audio_len, span_off, span_start,
+                                                    span_end, span_groups, ws, status);
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    dim3 grid_map((unsigned)((stride + kMapThreads - 1) / kMapThreads), (unsigned)B);
+    slot_map_kernel<<<grid_map, kMapThreads, 0, stream>>>(stride, keep_bg, in_len, audio_begin, audio_len, span_off,
+                                                          span_start, span_end, span_groups, ws, slot_map);
+    return cudaGetLastError();
+}
+
 }  // namespace
 
 size_t anchor_fuse_workspace_bytes(const voxzip_cache_desc &d, int32_t prefill_stride, int32_t num_spans) {
@@ -275,16 +425,9 @@ cudaError_t launch_anchor_fuse(const voxzip_cache_desc &d, const void *k_prefill
                                int32_t *status, cudaStream_t stream) {
     FuseWorkspace ws;
     carve(d, prefill_stride, num_spans, static_cast<char *>(workspace), &ws);
-    const bool has_anchor = anchor_k != nullptr;
-    span_scan_kernel<<<d.batch, kScanThreads, 0, stream>>>(
-        d.batch, prefill_stride, d.capacity, num_spans, anchor_stride, has_anchor, in_len, audio_begin,
-        audio_len, span_off, span_start, span_end, span_groups, ws, status);
-    cudaError_t err = cudaGetLastError();
-    if (err != cudaSuccess) return err;
-    dim3 grid_map((unsigned)((prefill_stride + kMapThreads - 1) / kMapThreads), (unsigned)d.batch);
-    slot_map_kernel<<<grid_map, kMapThreads, 0, stream>>>(prefill_stride, in_len, span_off, span_start,
-                                                          span_end, span_groups, ws, slot_map);
-    err = cudaGetLastError();
+    cudaError_t err = launch_slot_plan(d.batch, d.capacity, prefill_stride, num_spans, anchor_stride,
+                                       anchor_k != nullptr, true, in_len, audio_begin, audio_len, span_off,
+                                       span_start, span_end, span_groups, ws, slot_map, status, stream);
     if (err != cudaSuccess) return err;
     const bool bf16 = d.dtype == VOXZIP_BF16;
     if (d.head_dim == 128)
@@ -299,6 +442,38 @@ cudaError_t launch_anchor_fuse(const voxzip_cache_desc &d, const void *k_prefill
                                                        stream)
                 : launch_fuse_rows<float, 64>(d, prefill_stride, anchor_stride, k_prefill, v_prefill, anchor_k,
                                               anchor_v, ws, k_cache, v_cache, score, pos, len, stream);
+}
+
+size_t embed_fuse_workspace_bytes(int32_t batch, int32_t stride, int32_t num_spans) {
+    voxzip_cache_desc d{};
+    d.batch = batch;
+    return carve(d, stride, num_spans, nullptr, nullptr);
+}
+
+cudaError_t launch_embed_fuse(int32_t B, int32_t D, int32_t C, bool bf16, const void *e_in, int32_t stride,
+                              const int32_t *in_len, const int32_t *audio_begin, const int32_t *audio_len,
+                              const int32_t *span_off, int32_t num_spans, const int32_t *span_start,
+                              const int32_t *span_end, const int32_t *span_groups, const void *e_text,
+                              int32_t text_stride, bool keep_background, void *e_out, int32_t *pos, int32_t *len,
+                              int32_t *slot_map, void *workspace, int32_t *status, cudaStream_t stream) {
+    voxzip_cache_desc d{};
+    d.batch = B;
+    FuseWorkspace ws;
+    carve(d, stride, num_spans, static_cast<char *>(workspace), &ws);
+    cudaError_t err = launch_slot_plan(B, C, stride, num_spans, text_stride, e_text != nullptr, keep_background,
+                                       in_len, audio_begin, audio_len, span_off, span_start, span_end, span_groups,
+                                       ws, slot_map, status, stream);
+    if (err != cudaSuccess) return err;
+    dim3 grid((unsigned)((stride + kWideWarps - 1) / kWideWarps), (unsigned)B);
+    if (bf16)
+        fuse_wide_kernel<__nv_bfloat16><<<grid, kWideWarps * 32, 0, stream>>>(
+            C, stride, D, text_stride, (const __nv_bfloat16 *)e_in, (const __nv_bfloat16 *)e_text, ws,
+            (__nv_bfloat16 *)e_out, pos, len);
+    else
+        fuse_wide_kernel<float><<<grid, kWideWarps * 32, 0, stream>>>(C, stride, D, text_stride, (const float *)e_in,
+                                                                      (const float *)e_text, ws, (float *)e_out, pos,
+                                                                      len);
+    return cudaGetLastError();
 }
 
 }  // namespace voxzip

@@ -3,6 +3,7 @@
 #include <math.h>
 
 #include "common.cuh"
+#include "embed.cuh"
 
 namespace {
 
@@ -101,6 +102,87 @@ voxzip_status voxzip_anchor_fuse(const voxzip_cache_desc *desc, const void *k_pr
         *desc, k_prefill, v_prefill, prefill_stride, in_len, audio_begin, audio_len, span_off, num_spans,
         span_start, span_end, span_groups, anchor_k, anchor_v, anchor_stride, k_cache, v_cache, score, pos, len,
         slot_map, workspace, status, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+voxzip_status voxzip_segments_to_spans(int32_t n, const double *t_start, const double *t_end,
+                                       const double *confidence, const int32_t *text_len,
+                                       double tau_total, int32_t audio_len, int32_t audio_begin,
+                                       double threshold, int32_t *span_start, int32_t *span_end,
+                                       int32_t *span_groups, int32_t *seg_index,
+                                       int32_t *num_spans) {
+    if (n < 0 || !num_spans || !(tau_total > 0.0) || isinf(tau_total) || audio_len < 0 || audio_begin < 0 ||
+        (int64_t)audio_begin + audio_len > INT32_MAX)
+        return VOXZIP_EINVAL;
+    if (n > 0 && (!t_start || !t_end || !confidence || !text_len || !span_start || !span_end || !span_groups ||
+                  !seg_index))
+        return VOXZIP_EINVAL;
+    for (int32_t i = 0; i < n; ++i)
+        if (!(t_end[i] >= t_start[i]) || text_len[i] < 1 || (i > 0 && !(t_start[i] >= t_start[i - 1])))
+            return VOXZIP_EINVAL;
+    // Eq. 3 on one time: floor(L_a * (t / tau_total)) clamped to the audio.
+    auto index_of = [&](double t) -> int64_t {
+        const double f = floor((double)audio_len * (t / tau_total));
+        if (!(f > 0.0)) return 0;  // also NaN
+        return f >= (double)audio_len ? audio_len : (int64_t)f;
+    };
+    int32_t out = 0;
+    int64_t end_prev = 0;
+    for (int32_t i = 0; i < n; ++i) {
+        if (!(confidence[i] > threshold)) continue;  // the confidence filter
+        int64_t a = index_of(t_start[i]), b = index_of(t_end[i]);
+        a = a < end_prev ? end_prev : a;
+        b = b < a ? a : b;
+        span_start[out] = (int32_t)(audio_begin + a);
+        span_end[out] = (int32_t)(audio_begin + b);
+        span_groups[out] = text_len[i];
+        seg_index[out] = i;
+        end_prev = b;
+        ++out;
+    }
+    *num_spans = out;
+    return VOXZIP_OK;
+}
+
+namespace {
+bool embed_desc_ok(const voxzip_embed_desc *d) {
+    if (d == nullptr || d->batch < 1 || d->d_model < 1 || d->capacity < 1) return false;
+    if (d->dtype != VOXZIP_F32 && d->dtype != VOXZIP_BF16) return false;
+    const int elems16 = d->dtype == VOXZIP_BF16 ? 8 : 4;  // elements per 16-byte vector
+    return d->d_model % elems16 == 0;
+}
+}  // namespace
+
+size_t voxzip_embed_fuse_workspace_size(const voxzip_embed_desc *desc, int32_t stride, int32_t num_spans) {
+    if (!embed_desc_ok(desc) || stride < 1 || num_spans < 0) return 0;
+    return voxzip::embed_fuse_workspace_bytes(desc->batch, stride, num_spans);
+}
+
+voxzip_status voxzip_embed_fuse(const voxzip_embed_desc *desc, const void *e_in, int32_t stride,
+                                const int32_t *in_len, const int32_t *audio_begin,
+                                const int32_t *audio_len, const int32_t *span_off,
+                                int32_t num_spans, const int32_t *span_start,
+                                const int32_t *span_end, const int32_t *span_groups,
+                                const void *e_text, int32_t text_stride, int32_t keep_background,
+                                void *e_out, int32_t *pos, int32_t *len, int32_t *slot_map,
+                                void *workspace, size_t workspace_bytes, voxzip_stream_t stream) {
+    if (!embed_desc_ok(desc) || stride < 1 || num_spans < 0) return VOXZIP_EINVAL;
+    if (!e_in || !in_len || !audio_begin || !audio_len || !span_off || !e_out || !pos || !len || !workspace)
+        return VOXZIP_EINVAL;
+    if (num_spans > 0 && (!span_start || !span_end || !span_groups)) return VOXZIP_EINVAL;
+    if (e_text && text_stride < 1) return VOXZIP_EINVAL;
+    if (keep_background != 0 && keep_background != 1) return VOXZIP_EINVAL;
+    if (!aligned16(e_in) || !aligned16(e_out) || (e_text && !aligned16(e_text))) return VOXZIP_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return VOXZIP_EINVAL;
+    if (workspace_bytes < voxzip::embed_fuse_workspace_bytes(desc->batch, stride, num_spans)) return VOXZIP_EINVAL;
+    if (desc->batch > kMaxGridY) return VOXZIP_EUNSUPPORTED;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    return from_cuda(voxzip::launch_embed_fuse(desc->batch, desc->d_model, desc->capacity,
+                                               desc->dtype == VOXZIP_BF16, e_in, stride, in_len, audio_begin,
+                                               audio_len, span_off, num_spans, span_start, span_end, span_groups,
+                                               e_text, text_stride, keep_background != 0, e_out, pos, len, slot_map,
+                                               workspace, status, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 voxzip_status voxzip_decode_step(const voxzip_cache_desc *desc, int32_t layer_begin,

@@ -336,3 +336,125 @@ def unit_inputs_cpu(w: Workload, spans: Spans, b: int, l: int, h: int, steps=Non
                 audio_len=w.audio_len[b], span_start=st, span_end=en, span_groups=gr,
                 q=f64(torch.stack(qs)), k_new=f64(torch.stack(kns)), v_new=f64(torch.stack(vns)),
                 new_pos=np.array([w.in_len[b] + t for t in range(S)], np.int32))
+
+
+# ----------------------------------------------------------------------------- embedding level
+
+@dataclass(frozen=True)
+class EmbedWorkload:
+    """Stage 1 where the paper runs it: prompt embeddings [B][in_len][d_model] with an audio region,
+    and the ASR output of that audio as timed segments.
+
+    Recipe: the prompt is text_len // 8 text tokens, the audio tokens (12.5 per second, as the
+    Qwen3-Omni audio encoder emits), then the rest of the text. The audio is cut left to right
+    into ASR segments of U[seg_sec] seconds separated, with probability gap_prob, by silences of
+    U[gap_sec] seconds; segment times are the token boundaries jittered by up to +-jitter_tok
+    tokens (so the floor of Eq. 3 matters) and kept sorted; a segment's transcription has
+    L_t = max(1, round(text_per_sec x duration)) tokens (about 0.26 text tokens per audio token,
+    the paper's ~0.25x); its confidence is U(0, 0.3) with probability low_conf_prob, else
+    U(0.3, 1). Embeddings are N(0, 1) (audio) and 0.5 N(0, 1) (text) rounded to the dtype; text
+    embeddings are drawn for every segment, kept or not, in segment order."""
+    name: str
+    batch: int
+    audio_len: tuple
+    text_len: int
+    d_model: int
+    dtype: torch.dtype = torch.bfloat16
+    rate: float = 12.5
+    seg_sec: tuple = (2.0, 10.0)
+    gap_prob: float = 0.1
+    gap_sec: tuple = (0.5, 3.0)
+    jitter_tok: float = 0.4
+    text_per_sec: float = 3.2
+    low_conf_prob: float = 0.1
+    seed: int = 0
+    description: str = field(default="", compare=False)
+
+    @property
+    def in_len(self) -> tuple:
+        return tuple(a + self.text_len for a in self.audio_len)
+
+    @property
+    def audio_begin(self) -> int:
+        return self.text_len // 8
+
+    @property
+    def stride(self) -> int:
+        return max(self.in_len)
+
+    @property
+    def capacity(self) -> int:
+        return self.stride
+
+
+def _make_embed_configs():
+    c = {}
+    c["embed_tiny"] = EmbedWorkload("embed_tiny", batch=2, audio_len=(600, 430), text_len=32, d_model=256,
+                                    dtype=torch.float32, seed=10, description="2 clips, d 256, fp32")
+    c["embed_short"] = EmbedWorkload("embed_short", batch=1, audio_len=(375,), text_len=256, d_model=2048,
+                                     seed=11, description="30 s clip, d 2048, bf16")
+    c["embed_stress"] = EmbedWorkload("embed_stress", batch=4, audio_len=(45000,) * 4, text_len=1024, d_model=2048,
+                                      seed=12, description="4 x 60 min audio, d 2048, bf16")
+    return c
+
+
+EMBED_CONFIGS = _make_embed_configs()
+
+
+@dataclass
+class Segments:
+    """ASR output of one sequence: per segment start / end time (s), confidence, text tokens."""
+    t_start: np.ndarray
+    t_end: np.ndarray
+    confidence: np.ndarray
+    text_len: np.ndarray
+    tau_total: float
+
+
+def make_segments(w: EmbedWorkload) -> list:
+    rng = np.random.default_rng(3000 + w.seed)
+    out = []
+    for b in range(w.batch):
+        La = w.audio_len[b]
+        tau = La / w.rate
+        ts, te, cf, tl = [], [], [], []
+        t = 0.0
+        while t < tau:
+            if rng.random() < w.gap_prob:
+                t += float(rng.uniform(*w.gap_sec))
+                continue
+            dur = float(rng.uniform(*w.seg_sec))
+            e = min(tau, t + dur)
+            j0, j1 = rng.uniform(-w.jitter_tok, w.jitter_tok, 2) / w.rate
+            s_t = max(0.0, t + j0) if not ts else max(ts[-1], t + j0)
+            ts.append(s_t)
+            te.append(max(s_t, e + j1))
+            cf.append(float(rng.uniform(0.0, 0.3)) if rng.random() < w.low_conf_prob else float(rng.uniform(0.3, 1.0)))
+            tl.append(max(1, int(round(w.text_per_sec * (e - t)))))
+            t = e
+        out.append(Segments(np.asarray(ts), np.asarray(te), np.asarray(cf), np.asarray(tl, np.int32), tau))
+    return out
+
+
+_E, _ET = 7, 8   # stream kinds of the embedding level
+
+
+def make_embeddings(w: EmbedWorkload, device="cpu"):
+    """Prompt embeddings [B][stride][d_model] in the dtype; rows past in_len are zero."""
+    e = torch.zeros(w.batch, w.stride, w.d_model, dtype=w.dtype, device=device)
+    for b in range(w.batch):
+        n = w.in_len[b]
+        e[b, :n] = torch.randn(n, w.d_model, generator=_gen(w, device, _E, b), device=device).to(w.dtype)
+    return e
+
+
+def make_text_embeddings(w: EmbedWorkload, segments: list, device="cpu"):
+    """Embedded transcriptions of every segment, [B][max rows][d_model]: sequence b's segments'
+    text tokens concatenated in segment order (rows past them zero)."""
+    rows = [int(s.text_len.sum()) for s in segments]
+    t = torch.zeros(w.batch, max(1, max(rows)), w.d_model, dtype=w.dtype, device=device)
+    for b in range(w.batch):
+        if rows[b]:
+            x = torch.randn(rows[b], w.d_model, generator=_gen(w, device, _ET, b), device=device)
+            t[b, :rows[b]] = (0.5 * x).to(w.dtype)
+    return t
