@@ -102,13 +102,20 @@ class Oracle:
                                         _F64P, _F64P, _i32, _f64, _f64, _F64P]
         lib.vzo_evict.argtypes = [_i32, _I32P, _i32, _i32, _f32, _F64P, _F64P, _F64P, _I32P,
                                   _F64P, _I32P]
+        lib.vzo_evict_ex.argtypes = [_i32, _I32P, _i32, _i32, _f32, _i32, _i32, _F64P, _F64P, _F64P,
+                                     _I32P, _F64P, _I32P]
         lib.vzo_run_unit.argtypes = [_i32, _i32, _i32, _i32, _I32P, _I32P, _I32P, _i32, _F64P,
                                      _F64P, _F64P, _F64P, _i32, _i32, _i32, _i32, _F64P, _F64P,
                                      _F64P, _I32P, _f64, _f64, _i32, _i32, _i32, _f32, _F64P,
                                      _F64P, _I32P, _I32P, _F64P, _F64P, _F64P, _F64P, _I32P,
                                      _I32P, _I32P, _I32P]
+        lib.vzo_run_unit_ex.argtypes = [_i32, _i32, _i32, _i32, _I32P, _I32P, _I32P, _i32, _F64P,
+                                     _F64P, _F64P, _F64P, _i32, _i32, _i32, _i32, _F64P, _F64P,
+                                     _F64P, _I32P, _f64, _f64, _i32, _i32, _i32, _f32, _i32, _i32, _F64P,
+                                     _F64P, _I32P, _I32P, _F64P, _F64P, _F64P, _F64P, _I32P,
+                                     _I32P, _I32P, _I32P]
         for f in (lib.vzo_stage1, lib.vzo_stage1_ex, lib.vzo_segments_to_spans, lib.vzo_decode_step,
-                  lib.vzo_evict, lib.vzo_run_unit):
+                  lib.vzo_evict, lib.vzo_evict_ex, lib.vzo_run_unit, lib.vzo_run_unit_ex):
             f.restype = ctypes.c_int
         self.lib = lib
         self.path = path
@@ -182,14 +189,18 @@ class Oracle:
         cache.n = int(n[0])
         return out
 
-    def evict(self, cache: UnitCache, budget: int, sink: int = 4, recent_frac: float = 0.2):
-        """Eq. 7-9 for one unit, in place. Returns (margin, kept flags of the pre-eviction slots)."""
+    def evict(self, cache: UnitCache, budget: int, sink: int = 4, recent_frac: float = 0.2, *,
+              history: bool = True, fill: bool = False):
+        """Eq. 7-9 for one unit, in place. history=False keeps sinks and a recent window only
+        (StreamingLLM); fill=True selects sinks / recents by position and fills the evicted slots
+        with the kept rows beyond the budget. Returns (margin, kept flags of the pre-eviction slots)."""
         n = np.array([cache.n], np.int32)
         margin = np.zeros(1)
         kept = np.zeros(max(cache.n, 1), np.int32)
-        rc = self.lib.vzo_evict(cache.D, _p(n, _I32P), int(budget), int(sink), float(recent_frac),
-                                _p(cache.K, _F64P), _p(cache.V, _F64P), _p(cache.score, _F64P),
-                                _p(cache.pos, _I32P), _p(margin, _F64P), _p(kept, _I32P))
+        rc = self.lib.vzo_evict_ex(cache.D, _p(n, _I32P), int(budget), int(sink), float(recent_frac),
+                                   int(bool(history)), int(bool(fill)), _p(cache.K, _F64P), _p(cache.V, _F64P),
+                                   _p(cache.score, _F64P), _p(cache.pos, _I32P), _p(margin, _F64P),
+                                   _p(kept, _I32P))
         if rc != OK:
             raise OracleError("vzo_evict", rc)
         pre_n = cache.n
@@ -198,7 +209,8 @@ class Oracle:
 
     def run_unit(self, xk, xv, in_len, audio_begin, audio_len, span_start, span_end, span_groups,
                  *, q, k_new, v_new, new_pos, gamma, scale, interval, budget, sink=4,
-                 recent_frac=0.2, capacity, anchor_k=None, anchor_v=None, cache_is_bf16=False):
+                 recent_frac=0.2, capacity, anchor_k=None, anchor_v=None, cache_is_bf16=False,
+                 history=True, fill=False):
         """Stage 1, then len(q) decode steps with an eviction every ``interval`` steps.
 
         q [steps][G][D]; k_new, v_new [steps][D]; new_pos [steps]. Returns a dict with ``out``,
@@ -225,12 +237,13 @@ class Oracle:
         stage1_len = np.zeros(1, np.int32)
         ak = None if anchor_k is None else _f64a(anchor_k)
         av = None if anchor_v is None else _f64a(anchor_v)
-        rc = self.lib.vzo_run_unit(
+        rc = self.lib.vzo_run_unit_ex(
             int(in_len), int(audio_begin), int(audio_len), len(ss), _p(ss, _I32P), _p(se, _I32P),
             _p(sg, _I32P), D, _p(xk, _F64P), _p(xv, _F64P), _p(ak, _F64P), _p(av, _F64P),
             int(bool(cache_is_bf16)), G, int(capacity), steps, _p(q, _F64P), _p(k_new, _F64P),
             _p(v_new, _F64P), _p(new_pos, _I32P), float(gamma), float(scale), int(interval),
-            int(budget), int(sink), float(recent_frac), _p(out, _F64P), _p(score_before, _F64P),
+            int(budget), int(sink), float(recent_frac), int(bool(history)), int(bool(fill)),
+            _p(out, _F64P), _p(score_before, _F64P),
             _p(len_before, _I32P), _p(kept_pos, _I32P), _p(margin, _F64P), _p(K, _F64P),
             _p(V, _F64P), _p(score, _F64P), _p(pos, _I32P), _p(n_final, _I32P),
             _p(slot_map, _I32P), _p(stage1_len, _I32P))

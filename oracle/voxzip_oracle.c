@@ -21,6 +21,11 @@
  *                    Sec. 3.2.2: temporally decayed accumulated score (Eq. 6).
  *   vzo_evict        Sec. 3.2.2: T attention sinks, a recent window of 20 % of the budget,
  *                    top-N history by decayed score, concatenation (Eq. 7-9).
+ *   vzo_evict_ex     the same selection as a policy: without history (the StreamingLLM baseline
+ *                    of Sec. 4), and with sinks / recents chosen by position and the kept rows
+ *                    beyond the budget filling the evicted slots (a compaction that moves at most
+ *                    n - budget rows; the kept set is the same as the ordered one on a cache in
+ *                    time order).
  *   vzo_run_unit     the three above in the paper's order for one unit: stage 1 at prefill,
  *                    then decode steps with an eviction every `interval` steps.
  * Every function is pinned by the CPU tests (closed forms, invariants, brute force and
@@ -327,27 +332,47 @@ static int candidate_order(const void *a, const void *b)
     return (x->pos > y->pos) - (x->pos < y->pos);
 }
 
+static int position_order(const void *a, const void *b)
+{
+    const vzo_candidate *x = (const vzo_candidate *)a;
+    const vzo_candidate *y = (const vzo_candidate *)b;
+    return (x->pos > y->pos) - (x->pos < y->pos);
+}
+
 /*
- * Budgeted eviction for one unit (Sec. 3.2.2, Eq. 7-9). If the cache holds more than `budget`
- * rows it keeps the first T = sink rows, the last M = floor(budget * recent_frac) rows and the
- * N = budget - T - M history rows of [T, n - M) with the highest decayed score, then moves the
- * kept rows (K, V, score, pos together) to [0, budget) in ascending slot order.
+ * Budgeted eviction for one unit (Sec. 3.2.2, Eq. 7-9), with the policy variants of the same
+ * selection. If the cache holds more than `budget` rows it keeps T = sink attention sinks, a
+ * recent window of M rows and the N = budget - T - M history rows with the highest decayed score.
  *
+ *   history = 1   M = floor(budget * recent_frac): VoxZip's top-N history (Eq. 9)
+ *   history = 0   M = budget - T, N = 0: sinks and a recent window only (the StreamingLLM policy
+ *                 the paper compares against)
+ *   fill = 0      sinks are the first T slots, the recent window the last M slots, candidates
+ *                 the slots between; the kept rows move to [0, budget) in ascending slot order
+ *                 (Eq. 7-8 as concatenation in order)
+ *   fill = 1      the same sets chosen by position instead of slot (sinks: the T lowest
+ *                 positions, recent: the M highest), so the cache need not be in time order;
+ *                 kept rows already below `budget` stay where they are and the kept rows at
+ *                 slots >= budget fill the evicted slots below it, both taken in ascending slot
+ *                 order. On a cache in time order both modes keep the same rows.
+ * Ties in the top-N go to the lower position. K, V, score and pos move together.
  *   margin  score of the N-th kept history row minus that of the best evicted one (+inf when
  *           there is no such pair or nothing is evicted); parity tests gate on it
  *   kept    if non-NULL, [n] flags: 1 for every slot kept (before the move)
  */
-int vzo_evict(int32_t D, int32_t *n_io, int32_t budget, int32_t sink, float recent_frac,
-              double *K, double *V, double *score, int32_t *pos, double *margin, int32_t *kept)
+int vzo_evict_ex(int32_t D, int32_t *n_io, int32_t budget, int32_t sink, float recent_frac,
+                 int32_t history, int32_t fill, double *K, double *V, double *score, int32_t *pos,
+                 double *margin, int32_t *kept)
 {
     const int32_t n = *n_io;
     *margin = INFINITY;
-    if (budget < 0 || sink < 0 || D <= 0 || !(recent_frac >= 0.0f && recent_frac <= 1.0f))
+    if (budget < 0 || sink < 0 || D <= 0 || !(recent_frac >= 0.0f && recent_frac <= 1.0f) ||
+        (history != 0 && history != 1) || (fill != 0 && fill != 1))
         return VZO_EINVAL;
-    const int32_t M = (int32_t)floor((double)recent_frac * (double)budget);
     const int32_t T = sink;
+    const int32_t M = history ? (int32_t)floor((double)recent_frac * (double)budget) : budget - T;
     const int32_t N = budget - T - M;
-    if (N < 0)
+    if (N < 0 || M < 0)
         return VZO_EINVAL;
     if (kept)
         for (int32_t j = 0; j < n; ++j)
@@ -355,49 +380,80 @@ int vzo_evict(int32_t D, int32_t *n_io, int32_t budget, int32_t sink, float rece
     if (n <= budget)
         return VZO_OK;
 
-    /* Eq. 9: I_hist = Top_N(A^(t)[T : -M]). */
-    const int32_t nc = n - M - T;
-    vzo_candidate *c = (vzo_candidate *)malloc(sizeof(vzo_candidate) * (size_t)nc);
+    vzo_candidate *all = (vzo_candidate *)malloc(sizeof(vzo_candidate) * (size_t)n);
     int32_t *keep = (int32_t *)calloc((size_t)n, sizeof(int32_t));
-    if (!c || !keep) {
-        free(c);
+    if (!all || !keep) {
+        free(all);
         free(keep);
         return VZO_ENOMEM;
     }
-    for (int32_t j = 0; j < nc; ++j) {
-        c[j].score = score[T + j];
-        c[j].pos = pos[T + j];
-        c[j].slot = T + j;
+    /* The slots in the order that defines "first" and "last": slot order, or time (position). */
+    for (int32_t j = 0; j < n; ++j) {
+        all[j].score = score[j];
+        all[j].pos = pos[j];
+        all[j].slot = j;
     }
+    if (fill)
+        qsort(all, (size_t)n, sizeof(vzo_candidate), position_order);
+    for (int32_t r = 0; r < T; ++r)
+        keep[all[r].slot] = 1;
+    for (int32_t r = n - M; r < n; ++r)
+        keep[all[r].slot] = 1;
+    /* Eq. 9: I_hist = Top_N over the rows between the sinks and the recent window. */
+    const int32_t nc = n - M - T;
+    vzo_candidate *c = all + T;
     qsort(c, (size_t)nc, sizeof(vzo_candidate), candidate_order);
     if (N >= 1 && N < nc)
         *margin = c[N - 1].score - c[N].score;
-    for (int32_t j = 0; j < T; ++j)
-        keep[j] = 1;
-    for (int32_t j = 0; j < N; ++j)
-        keep[c[j].slot] = 1;
-    for (int32_t j = n - M; j < n; ++j)
-        keep[j] = 1;
-
-    /* Eq. 7-8: concatenate sinks, selected history and recent rows, preserving their order. */
-    int32_t w = 0;
-    for (int32_t j = 0; j < n; ++j) {
-        if (kept)
+    for (int32_t r = 0; r < N; ++r)
+        keep[c[r].slot] = 1;
+    if (kept)
+        for (int32_t j = 0; j < n; ++j)
             kept[j] = keep[j];
-        if (!keep[j])
-            continue;
-        if (w != j) {
-            memmove(K + (int64_t)w * D, K + (int64_t)j * D, sizeof(double) * (size_t)D);
-            memmove(V + (int64_t)w * D, V + (int64_t)j * D, sizeof(double) * (size_t)D);
-            score[w] = score[j];
-            pos[w] = pos[j];
+
+    if (!fill) {
+        /* Eq. 7-8: concatenate sinks, selected history and recent rows, preserving their order. */
+        int32_t w = 0;
+        for (int32_t j = 0; j < n; ++j) {
+            if (!keep[j])
+                continue;
+            if (w != j) {
+                memmove(K + (int64_t)w * D, K + (int64_t)j * D, sizeof(double) * (size_t)D);
+                memmove(V + (int64_t)w * D, V + (int64_t)j * D, sizeof(double) * (size_t)D);
+                score[w] = score[j];
+                pos[w] = pos[j];
+            }
+            ++w;
         }
-        ++w;
+    } else {
+        /* Hole filling: kept rows at slots >= budget go, in slot order, to the evicted slots
+           below budget, in slot order. There are as many of each. */
+        int32_t h = 0;
+        for (int32_t j = budget; j < n; ++j) {
+            if (!keep[j])
+                continue;
+            while (h < budget && keep[h])
+                ++h;
+            if (h >= budget)
+                break; /* cannot happen: the kept rows number exactly `budget` */
+            memcpy(K + (int64_t)h * D, K + (int64_t)j * D, sizeof(double) * (size_t)D);
+            memcpy(V + (int64_t)h * D, V + (int64_t)j * D, sizeof(double) * (size_t)D);
+            score[h] = score[j];
+            pos[h] = pos[j];
+            ++h;
+        }
     }
-    free(c);
+    free(all);
     free(keep);
-    *n_io = w; /* == budget */
+    *n_io = budget;
     return VZO_OK;
+}
+
+/* VoxZip's eviction (history = 1) with ordered compaction. */
+int vzo_evict(int32_t D, int32_t *n_io, int32_t budget, int32_t sink, float recent_frac,
+              double *K, double *V, double *score, int32_t *pos, double *margin, int32_t *kept)
+{
+    return vzo_evict_ex(D, n_io, budget, sink, recent_frac, 1, 0, K, V, score, pos, margin, kept);
 }
 
 /*
@@ -417,16 +473,16 @@ int vzo_evict(int32_t D, int32_t *n_io, int32_t budget, int32_t sink, float rece
  *   slot_map     [in_len]                    stage-1 slot of every prefill token
  *   stage1_len                               cache length after stage 1
  */
-int vzo_run_unit(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t n_spans,
-                 const int32_t *span_start, const int32_t *span_end, const int32_t *span_groups,
-                 int32_t D, const double *xk, const double *xv, const double *anchor_k,
-                 const double *anchor_v, int32_t cache_is_bf16, int32_t G, int32_t capacity,
-                 int32_t steps, const double *q, const double *k_new, const double *v_new,
-                 const int32_t *new_pos, double gamma, double scale, int32_t interval,
-                 int32_t budget, int32_t sink, float recent_frac, double *out,
-                 double *score_before, int32_t *len_before, int32_t *kept_pos, double *margin,
-                 double *K, double *V, double *score, int32_t *pos, int32_t *n_final,
-                 int32_t *slot_map, int32_t *stage1_len)
+int vzo_run_unit_ex(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t n_spans,
+                    const int32_t *span_start, const int32_t *span_end, const int32_t *span_groups,
+                    int32_t D, const double *xk, const double *xv, const double *anchor_k,
+                    const double *anchor_v, int32_t cache_is_bf16, int32_t G, int32_t capacity,
+                    int32_t steps, const double *q, const double *k_new, const double *v_new,
+                    const int32_t *new_pos, double gamma, double scale, int32_t interval,
+                    int32_t budget, int32_t sink, float recent_frac, int32_t history, int32_t fill,
+                    double *out, double *score_before, int32_t *len_before, int32_t *kept_pos,
+                    double *margin, double *K, double *V, double *score, int32_t *pos,
+                    int32_t *n_final, int32_t *slot_map, int32_t *stage1_len)
 {
     if (interval <= 0 || steps < 0)
         return VZO_EINVAL;
@@ -464,7 +520,8 @@ int vzo_run_unit(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t
             for (int32_t j = 0; j < capacity; ++j)
                 score_before[(int64_t)ev * capacity + j] = j < n ? score[j] : 0.0;
             len_before[ev] = n;
-            rc = vzo_evict(D, &n, budget, sink, recent_frac, K, V, score, pos, &margin[ev], NULL);
+            rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,
+                              &margin[ev], NULL);
             if (rc != VZO_OK)
                 return rc;
             for (int32_t j = 0; j < budget; ++j)
@@ -474,4 +531,23 @@ int vzo_run_unit(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t
     }
     *n_final = n;
     return VZO_OK;
+}
+
+/* The whole path with VoxZip's eviction and ordered compaction. */
+int vzo_run_unit(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t n_spans,
+                 const int32_t *span_start, const int32_t *span_end, const int32_t *span_groups,
+                 int32_t D, const double *xk, const double *xv, const double *anchor_k,
+                 const double *anchor_v, int32_t cache_is_bf16, int32_t G, int32_t capacity,
+                 int32_t steps, const double *q, const double *k_new, const double *v_new,
+                 const int32_t *new_pos, double gamma, double scale, int32_t interval,
+                 int32_t budget, int32_t sink, float recent_frac, double *out,
+                 double *score_before, int32_t *len_before, int32_t *kept_pos, double *margin,
+                 double *K, double *V, double *score, int32_t *pos, int32_t *n_final,
+                 int32_t *slot_map, int32_t *stage1_len)
+{
+    return vzo_run_unit_ex(in_len, audio_begin, audio_len, n_spans, span_start, span_end,
+                           span_groups, D, xk, xv, anchor_k, anchor_v, cache_is_bf16, G, capacity,
+                           steps, q, k_new, v_new, new_pos, gamma, scale, interval, budget, sink,
+                           recent_frac, 1, 0, out, score_before, len_before, kept_pos, margin, K,
+                           V, score, pos, n_final, slot_map, stage1_len);
 }

@@ -498,6 +498,104 @@ def pin_evict_invariants(orc):
         raise AssertionError("budget below T + M accepted")
 
 
+def pin_evict_fill_hand(orc):
+    """Hand-worked hole-filling eviction on a cache out of time order, the ordered eviction of the
+    same slots, and the StreamingLLM policy with hole filling."""
+    g = _golden("evict_fill_hand.json")
+    n, D = g["n"], 2
+    K = np.array([[j, 10.0 * j] for j in range(n)])
+    for key, kw in (("fill", dict(fill=True)), ("ordered", dict(fill=False)),
+                    ("streaming_fill", dict(fill=True, history=False))):
+        case = g[key]
+        c = O.UnitCache.from_rows(n, K, -K, g["pos"], g["score"])
+        margin, kept = orc.evict(c, g["budget"], sink=g["sink"], recent_frac=g["recent_frac"], **kw)
+        src = case["expected_src"]
+        assert c.n == g["budget"]
+        np.testing.assert_array_equal(c.pos[:c.n], case["expected_pos"])
+        np.testing.assert_array_equal(c.score[:c.n], np.array(g["score"])[src])
+        np.testing.assert_array_equal(c.K[:c.n], K[src])
+        np.testing.assert_array_equal(c.V[:c.n], -K[src])
+        assert margin == _num(case["expected_margin"]), (key, margin)
+        if "expected_kept" in case:
+            np.testing.assert_array_equal(kept.astype(int), case["expected_kept"])
+            np.testing.assert_array_equal(c.score[:c.n], case["expected_score"])
+
+
+def pin_evict_fill_matches_ordered_in_time_order(orc):
+    """On a cache in time order, hole filling keeps exactly the rows the ordered compaction keeps
+    (with and without history). It leaves every kept row below the budget in place, moves at most
+    n - budget rows, and each row moves with its K, V, score and position."""
+    rng = np.random.default_rng(11)
+    for trial in range(40):
+        D = 3
+        n = int(rng.integers(8, 200))
+        budget = int(rng.integers(5, n + 10))
+        frac = float(rng.choice([0.2, 0.1, 0.5]))
+        history = bool(rng.integers(0, 2))
+        M = math.floor(float(np.float32(frac)) * budget) if history else budget - 4
+        if budget - 4 - M < 0:
+            continue
+        K = rng.standard_normal((n, D))
+        score = rng.integers(0, 8, n) / 8.0
+        pos = np.sort(rng.choice(10 * n, n, replace=False)).astype(np.int32)
+        a = O.UnitCache.from_rows(n, K, 2 * K, pos, score)
+        b = O.UnitCache.from_rows(n, K, 2 * K, pos, score)
+        ma, ka = orc.evict(a, budget, recent_frac=frac, history=history)
+        mb, kb = orc.evict(b, budget, recent_frac=frac, history=history, fill=True)
+        assert a.n == b.n == min(n, budget) and ma == mb
+        np.testing.assert_array_equal(ka, kb)
+        np.testing.assert_array_equal(np.sort(b.pos[:b.n]), a.pos[:a.n])
+        src = np.searchsorted(pos, b.pos[:b.n])
+        np.testing.assert_array_equal(b.K[:b.n], K[src])
+        np.testing.assert_array_equal(b.V[:b.n], 2 * K[src])
+        np.testing.assert_array_equal(b.score[:b.n], score[src])
+        stay = kb[:b.n]
+        np.testing.assert_array_equal(src[stay], np.nonzero(stay)[0])
+        assert int((src != np.arange(b.n)).sum()) <= max(0, n - budget)
+
+
+def pin_evict_fill_bruteforce_scrambled(orc):
+    """Tiny caches whose slots are a random permutation of time order: hole filling keeps the set
+    brute-force search keeps on the time-ordered cache (sinks and recents by position, the best
+    N-subset of the rest with ties to lower positions)."""
+    rng = np.random.default_rng(12)
+    for trial in range(40):
+        n = int(rng.integers(6, 14))
+        budget = int(rng.integers(5, n))
+        M = math.floor(float(np.float32(0.2)) * budget)
+        N = budget - 4 - M
+        if N < 0:
+            continue
+        score = rng.integers(0, 4, n) / 4.0
+        pos = np.sort(rng.choice(1000, n, replace=False)).astype(np.int32)
+        expect = set(pos[_brute_force_keep(score, pos, 4, M, N)])
+        perm = rng.permutation(n)
+        c = O.UnitCache.from_rows(n, perm[:, None].astype(float), np.zeros((n, 1)), pos[perm], score[perm])
+        orc.evict(c, budget, fill=True)
+        assert set(c.pos[:c.n]) == expect
+        np.testing.assert_array_equal(pos[c.K[:c.n, 0].astype(int)], c.pos[:c.n])
+
+
+def pin_evict_streaming(orc):
+    """Without history the kept rows are the T lowest and the budget - T highest positions, in
+    either compaction (the StreamingLLM baseline)."""
+    rng = np.random.default_rng(13)
+    for trial in range(30):
+        n = int(rng.integers(6, 100))
+        budget = int(rng.integers(4, n + 5))
+        pos = rng.choice(5 * n, n, replace=False).astype(np.int32)
+        score = rng.random(n)
+        order = np.sort(pos)
+        expect = set(order[:4]) | set(order[n - (budget - 4):]) if n > budget else set(pos)
+        c = O.UnitCache.from_rows(n, np.zeros((n, 1)), np.zeros((n, 1)), pos, score)
+        margin, _ = orc.evict(c, budget, history=False, fill=True)
+        assert set(c.pos[:c.n]) == expect and margin == math.inf
+        srt = np.argsort(pos)
+        c = O.UnitCache.from_rows(n, np.zeros((n, 1)), np.zeros((n, 1)), pos[srt], score[srt])
+        orc.evict(c, budget, history=False)
+        assert set(c.pos[:c.n]) == expect
+
+
 # ----------------------------------------------------------------------------- whole unit
 
 def pin_run_unit_identity(orc):

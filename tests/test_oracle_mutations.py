@@ -46,10 +46,10 @@ MUTATIONS = [
      "if (x->score > y->score)\n        return 1;\n    if (x->score < y->score)\n        return -1;"),
     ("recent window rounded up", "floor((double)recent_frac * (double)budget)",
      "ceil((double)recent_frac * (double)budget)"),
-    ("recent window one short", "for (int32_t j = n - M; j < n; ++j)\n        keep[j] = 1;",
-     "for (int32_t j = n - M + 1; j < n; ++j)\n        keep[j] = 1;"),
-    ("sinks one short", "for (int32_t j = 0; j < T; ++j)\n        keep[j] = 1;",
-     "for (int32_t j = 0; j < T - 1; ++j)\n        keep[j] = 1;"),
+    ("recent window one short", "for (int32_t r = n - M; r < n; ++r)\n        keep[all[r].slot] = 1;",
+     "for (int32_t r = n - M + 1; r < n; ++r)\n        keep[all[r].slot] = 1;"),
+    ("sinks one short", "for (int32_t r = 0; r < T; ++r)\n        keep[all[r].slot] = 1;",
+     "for (int32_t r = 0; r < T - 1; ++r)\n        keep[all[r].slot] = 1;"),
     ("score not moved with its row", "score[w] = score[j];", "(void)0;"),
     ("position not moved with its row", "pos[w] = pos[j];", "(void)0;"),
     ("confidence filter keeps the threshold itself", "if (!(confidence[i] > threshold))",
@@ -64,6 +64,15 @@ MUTATIONS = [
      "} else if (0) {"),
     ("Partial drops the text too", "} else if (!keep_background && t >= audio_begin && t < audio_begin + audio_len) {",
      "} else if (!keep_background) {"),
+    ("hole filling picks sinks and recents by slot", "    if (fill)\n        qsort(all, (size_t)n, sizeof(vzo_candidate), position_order);\n", ""),
+    ("hole filling writes over kept rows", "while (h < budget && keep[h])", "while (h < budget && !keep[h])"),
+    ("hole filling leaves the score behind", "            score[h] = score[j];\n            pos[h] = pos[j];",
+     "            pos[h] = pos[j];"),
+    ("hole filling leaves the position behind", "            score[h] = score[j];\n            pos[h] = pos[j];",
+     "            score[h] = score[j];"),
+    ("StreamingLLM window one short", ": budget - T;", ": budget - T - 1;"),
+    ("history switch ignored", "history ? (int32_t)floor((double)recent_frac * (double)budget) : budget - T",
+     "(int32_t)floor((double)recent_frac * (double)budget)"),
     ("margin against the wrong runner-up", "*margin = c[N - 1].score - c[N].score;",
      "*margin = c[N - 1].score - c[N + 1 < nc ? N + 1 : N].score;"),
 ]
