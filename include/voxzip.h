@@ -61,6 +61,8 @@ typedef enum {
 #define VOXZIP_DEV_BAD_BUDGET 0x8u /* budget < sink + floor(budget * recent_frac); unit skipped */
 #define VOXZIP_DEV_TIMEOUT 0x10u   /* a bounded wait inside a kernel gave up; outputs of that unit
                                       are not valid (never expected; reported instead of hanging) */
+#define VOXZIP_DEV_BAD_POSITIONS 0x20u /* a unit's positions were not unique, so a hole-filling
+                                          eviction could not keep exactly `budget` rows */
 
 typedef enum { VOXZIP_F32 = 0, VOXZIP_BF16 = 1 } voxzip_dtype;
 
@@ -261,6 +263,42 @@ voxzip_status voxzip_evict(const voxzip_cache_desc *desc, int32_t layer_begin,
                            int32_t layer_count, void *k_cache, void *v_cache, float *score,
                            int32_t *pos, int32_t *len, const int32_t *budget, int32_t sink,
                            float recent_frac, voxzip_stream_t stream);
+
+typedef enum {
+    VOXZIP_COMPACT_ORDERED = 0, /* kept rows move to [0, budget) in slot order (Eq. 7-8) */
+    VOXZIP_COMPACT_FILL = 1     /* kept rows beyond the budget fill the evicted slots below it */
+} voxzip_compaction;
+
+typedef struct {
+    int32_t sink;            /* T, attention sinks kept (the paper uses 4) */
+    float recent_frac;       /* M = floor(budget * recent_frac) recent rows (the paper: 0.2) */
+    int32_t history;         /* 1: the top-N history by decayed score (VoxZip, Eq. 9);
+                                0: no history, M = budget - T (the StreamingLLM policy) */
+    int32_t budget_stride_b; /* the budget of unit (b, l, h) is                                */
+    int32_t budget_stride_l; /*   budget[b * budget_stride_b + l * budget_stride_l]            */
+                             /* (1, 0): one per sequence; (L, 1): [B][L], one per layer        */
+    int32_t compaction;      /* voxzip_compaction */
+} voxzip_evict_policy;
+
+/*
+ * Eviction under a policy: the same selection as voxzip_evict with the switches above.
+ *
+ * VOXZIP_COMPACT_FILL chooses the sinks as the T lowest positions and the recent window as the M
+ * highest, so the cache need not be kept in time order. Kept rows below the budget stay where
+ * they are; the kept rows at slots >= budget move, in ascending slot order, into the evicted
+ * slots below the budget, in ascending slot order. At most n - budget rows move, against up to
+ * `budget` for the ordered compaction. On a cache in time order both keep the same rows. The
+ * decode step does not depend on slot order. A unit's positions must be unique; otherwise it
+ * reports VOXZIP_DEV_BAD_POSITIONS.
+ *
+ * The budget array is device int32 and covers every index the strides reach for the layers
+ * evicted. Errors: VOXZIP_EINVAL for a NULL policy, sink < 0, recent_frac outside [0, 1],
+ * history or compaction outside their values, or a negative stride; otherwise as voxzip_evict.
+ */
+voxzip_status voxzip_evict_ex(const voxzip_cache_desc *desc, int32_t layer_begin,
+                              int32_t layer_count, void *k_cache, void *v_cache, float *score,
+                              int32_t *pos, int32_t *len, const int32_t *budget,
+                              const voxzip_evict_policy *policy, voxzip_stream_t stream);
 
 /*
  * Waits for `stream`, then returns the device status word of the current device in *bits

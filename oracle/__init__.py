@@ -112,7 +112,7 @@ class Oracle:
         lib.vzo_run_unit_ex.argtypes = [_i32, _i32, _i32, _i32, _I32P, _I32P, _I32P, _i32, _F64P,
                                      _F64P, _F64P, _F64P, _i32, _i32, _i32, _i32, _F64P, _F64P,
                                      _F64P, _I32P, _f64, _f64, _i32, _i32, _i32, _f32, _i32, _i32, _F64P,
-                                     _F64P, _I32P, _I32P, _F64P, _F64P, _F64P, _F64P, _I32P,
+                                     _F64P, _I32P, _I32P, _I32P, _F64P, _F64P, _F64P, _F64P, _I32P,
                                      _I32P, _I32P, _I32P]
         for f in (lib.vzo_stage1, lib.vzo_stage1_ex, lib.vzo_segments_to_spans, lib.vzo_decode_step,
                   lib.vzo_evict, lib.vzo_evict_ex, lib.vzo_run_unit, lib.vzo_run_unit_ex):
@@ -225,6 +225,7 @@ class Oracle:
         n_ev = steps // interval
         out = np.zeros((max(steps, 1), G, D))
         score_before = np.zeros((max(n_ev, 1), capacity))
+        pos_before = np.full((max(n_ev, 1), capacity), -1, np.int32)
         len_before = np.zeros(max(n_ev, 1), np.int32)
         kept_pos = np.full((max(n_ev, 1), max(budget, 1)), -1, np.int32)
         margin = np.zeros(max(n_ev, 1))
@@ -243,14 +244,14 @@ class Oracle:
             int(bool(cache_is_bf16)), G, int(capacity), steps, _p(q, _F64P), _p(k_new, _F64P),
             _p(v_new, _F64P), _p(new_pos, _I32P), float(gamma), float(scale), int(interval),
             int(budget), int(sink), float(recent_frac), int(bool(history)), int(bool(fill)),
-            _p(out, _F64P), _p(score_before, _F64P),
+            _p(out, _F64P), _p(score_before, _F64P), _p(pos_before, _I32P),
             _p(len_before, _I32P), _p(kept_pos, _I32P), _p(margin, _F64P), _p(K, _F64P),
             _p(V, _F64P), _p(score, _F64P), _p(pos, _I32P), _p(n_final, _I32P),
             _p(slot_map, _I32P), _p(stage1_len, _I32P))
         if rc != OK:
             raise OracleError("vzo_run_unit", rc)
         nf = int(n_final[0])
-        return dict(out=out[:steps], score_before=score_before[:n_ev],
+        return dict(out=out[:steps], score_before=score_before[:n_ev], pos_before=pos_before[:n_ev],
                     len_before=len_before[:n_ev], kept_pos=kept_pos[:n_ev], margin=margin[:n_ev],
                     K=K[:nf], V=V[:nf], score=score[:nf], pos=pos[:nf], n=nf,
                     slot_map=slot_map[:int(in_len)], stage1_len=int(stage1_len[0]))

@@ -465,6 +465,8 @@ int vzo_evict(int32_t D, int32_t *n_io, int32_t budget, int32_t sink, float rece
  * Outputs:
  *   out          [steps][G][D]
  *   score_before [steps/interval][capacity]  scores just before each eviction (0-padded)
+ *   pos_before   [steps/interval][capacity]  (run_unit_ex, may be NULL) positions just before
+ *                                            each eviction (-1 padded)
  *   len_before   [steps/interval]            cache length just before each eviction
  *   kept_pos     [steps/interval][budget]    positions of the rows after each eviction
  *                                            (-1 padded when the cache was within budget)
@@ -480,9 +482,9 @@ int vzo_run_unit_ex(int32_t in_len, int32_t audio_begin, int32_t audio_len, int3
                     int32_t steps, const double *q, const double *k_new, const double *v_new,
                     const int32_t *new_pos, double gamma, double scale, int32_t interval,
                     int32_t budget, int32_t sink, float recent_frac, int32_t history, int32_t fill,
-                    double *out, double *score_before, int32_t *len_before, int32_t *kept_pos,
-                    double *margin, double *K, double *V, double *score, int32_t *pos,
-                    int32_t *n_final, int32_t *slot_map, int32_t *stage1_len)
+                    double *out, double *score_before, int32_t *pos_before, int32_t *len_before,
+                    int32_t *kept_pos, double *margin, double *K, double *V, double *score,
+                    int32_t *pos, int32_t *n_final, int32_t *slot_map, int32_t *stage1_len)
 {
     if (interval <= 0 || steps < 0)
         return VZO_EINVAL;
@@ -517,8 +519,11 @@ int vzo_run_unit_ex(int32_t in_len, int32_t audio_begin, int32_t audio_len, int3
         if (rc != VZO_OK)
             return rc;
         if (t % interval == 0) {
-            for (int32_t j = 0; j < capacity; ++j)
+            for (int32_t j = 0; j < capacity; ++j) {
                 score_before[(int64_t)ev * capacity + j] = j < n ? score[j] : 0.0;
+                if (pos_before)
+                    pos_before[(int64_t)ev * capacity + j] = j < n ? pos[j] : -1;
+            }
             len_before[ev] = n;
             rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,
                               &margin[ev], NULL);
@@ -548,6 +553,6 @@ int vzo_run_unit(int32_t in_len, int32_t audio_begin, int32_t audio_len, int32_t
     return vzo_run_unit_ex(in_len, audio_begin, audio_len, n_spans, span_start, span_end,
                            span_groups, D, xk, xv, anchor_k, anchor_v, cache_is_bf16, G, capacity,
                            steps, q, k_new, v_new, new_pos, gamma, scale, interval, budget, sink,
-                           recent_frac, 1, 0, out, score_before, len_before, kept_pos, margin, K,
-                           V, score, pos, n_final, slot_map, stage1_len);
+                           recent_frac, 1, 0, out, score_before, NULL, len_before, kept_pos,
+                           margin, K, V, score, pos, n_final, slot_map, stage1_len);
 }

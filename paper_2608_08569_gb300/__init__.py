@@ -4,18 +4,20 @@ The three steps of the path (arxiv 2608.08569, Sec. 3.2):
   voxzip_anchor_fuse   stage-1 semantic-anchored fusion of the prefilled cache (Eq. 4-5)
   voxzip_decode_step   append + GQA attention + decayed accumulated score (Eq. 1, 2, 6)
   voxzip_evict         sinks + recent window + top-N history, compacted in place (Eq. 7-9)
+  voxzip_evict_ex      the same under a policy: per-layer budgets, no history (StreamingLLM),
+                       hole-filling compaction (at most n - budget rows move)
 Stage 1 where the paper runs it, on input embeddings from ASR output:
   voxzip_segments_to_spans   confidence filter + time-to-index map (Eq. 3), on the host
   voxzip_embed_fuse          the same fusion on [B][tokens][d_model] embeddings with text anchors
 """
 from ._native import (CacheDesc, EmbedDesc, VoxZipError, allocate_cache, lib, voxzip_anchor_fuse,
                       voxzip_anchor_fuse_noalloc, voxzip_anchor_fuse_workspace_size, voxzip_decode_step,
-                      voxzip_embed_fuse, voxzip_embed_fuse_workspace_size, voxzip_evict, voxzip_get_status,
-                      voxzip_segments_to_spans)
-from ._native import (DEV_BAD_BUDGET, DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_TIMEOUT, VOXZIP_ECUDA,
+                      voxzip_embed_fuse, voxzip_embed_fuse_workspace_size, voxzip_evict, voxzip_evict_ex,
+                      voxzip_get_status, voxzip_segments_to_spans)
+from ._native import (DEV_BAD_BUDGET, DEV_BAD_POSITIONS, DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_TIMEOUT, VOXZIP_ECUDA,
                       VOXZIP_EINVAL, VOXZIP_ESCRATCH, VOXZIP_EUNSUPPORTED, VOXZIP_OK)
 
-__all__ = ["CacheDesc", "EmbedDesc", "voxzip_embed_fuse", "voxzip_embed_fuse_workspace_size",
+__all__ = ["CacheDesc", "EmbedDesc", "voxzip_evict_ex", "DEV_BAD_POSITIONS", "voxzip_embed_fuse", "voxzip_embed_fuse_workspace_size",
            "voxzip_segments_to_spans", "VoxZipError", "allocate_cache", "lib", "voxzip_anchor_fuse", "voxzip_anchor_fuse_noalloc",
            "voxzip_anchor_fuse_workspace_size", "voxzip_decode_step", "voxzip_evict", "voxzip_get_status",
            "DEV_BAD_BUDGET", "DEV_BAD_SPANS", "DEV_CAPACITY", "DEV_LEN_HINT", "DEV_TIMEOUT", "VOXZIP_ECUDA",

@@ -17,6 +17,8 @@ from .build import LIB_PATH
 
 VOXZIP_OK, VOXZIP_EINVAL, VOXZIP_EUNSUPPORTED, VOXZIP_ECUDA, VOXZIP_ESCRATCH = 0, 1, 2, 3, 4
 DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_BAD_BUDGET, DEV_TIMEOUT = 0x1, 0x2, 0x4, 0x8, 0x10
+DEV_BAD_POSITIONS = 0x20
+VOXZIP_COMPACT_ORDERED, VOXZIP_COMPACT_FILL = 0, 1
 VOXZIP_F32, VOXZIP_BF16 = 0, 1
 
 _DTYPES = {torch.float32: VOXZIP_F32, torch.bfloat16: VOXZIP_BF16}
@@ -71,6 +73,12 @@ class EmbedDesc:
         return _EmbedDesc(self.batch, self.d_model, self.capacity, _DTYPES[self.dtype])
 
 
+class _EvictPolicy(ctypes.Structure):
+    _fields_ = [("sink", ctypes.c_int32), ("recent_frac", ctypes.c_float), ("history", ctypes.c_int32),
+                ("budget_stride_b", ctypes.c_int32), ("budget_stride_l", ctypes.c_int32),
+                ("compaction", ctypes.c_int32)]
+
+
 _lock = threading.Lock()
 _lib = None
 _vp = ctypes.c_void_p
@@ -101,6 +109,8 @@ def lib() -> ctypes.CDLL:
                                              _f32, _f32, _i32, _vp, _vp]
             L.voxzip_evict.argtypes = [_DP, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _f32, _vp]
             L.voxzip_get_status.argtypes = [ctypes.POINTER(ctypes.c_uint32), _vp]
+            L.voxzip_evict_ex.argtypes = [_DP, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp,
+                                          ctypes.POINTER(_EvictPolicy), _vp]
             L.voxzip_segments_to_spans.argtypes = [_i32, _vp, _vp, _vp, _vp, _f64, _i32, _i32, _f64, _vp, _vp, _vp,
                                                    _vp, _vp]
             L.voxzip_embed_fuse.argtypes = [_EP, _vp, _i32, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _i32,
@@ -111,7 +121,7 @@ def lib() -> ctypes.CDLL:
             L.voxzip_status_string.restype = ctypes.c_char_p
             L.voxzip_version.restype = _i32
             for f in (L.voxzip_anchor_fuse, L.voxzip_decode_step, L.voxzip_evict, L.voxzip_get_status,
-                      L.voxzip_segments_to_spans, L.voxzip_embed_fuse):
+                      L.voxzip_segments_to_spans, L.voxzip_embed_fuse, L.voxzip_evict_ex):
                 f.restype = _i32
             _lib = L
     return _lib
@@ -329,6 +339,30 @@ def voxzip_evict(desc: CacheDesc, layer_begin: int, layer_count: int, k_cache, v
     _check("voxzip_evict", lib().voxzip_evict(
         ctypes.byref(d), int(layer_begin), int(layer_count), _ptr(k_cache), _ptr(v_cache), _ptr(score), _ptr(pos),
         _ptr(len_), _ptr(budget), int(sink), float(recent_frac), _stream(stream)))
+
+
+def voxzip_evict_ex(desc: CacheDesc, layer_begin: int, layer_count: int, k_cache, v_cache, score, pos, len_,
+                    budget, *, sink: int = 4, recent_frac: float = 0.2, history: bool = True,
+                    compaction: str = "ordered", stream=None) -> None:
+    """Eviction under a policy. `budget` is [B] (one per sequence) or [B][L] (one per layer);
+    history=False is the StreamingLLM policy (sinks + a recent window of budget - sink rows);
+    compaction="fill" chooses sinks / recents by position and fills the evicted slots with the kept
+    rows beyond the budget (at most n - budget rows move)."""
+    _check_cache(desc, k_cache, v_cache, score, pos, len_)
+    if budget.dim() == 1:
+        _need(budget, "budget", torch.int32, (desc.batch,))
+        sb, sl = 1, 0
+    else:
+        _need(budget, "budget", torch.int32, (desc.batch, desc.layers))
+        sb, sl = desc.layers, 1
+    if compaction not in ("ordered", "fill"):
+        raise ValueError("compaction must be 'ordered' or 'fill'")
+    pol = _EvictPolicy(int(sink), float(recent_frac), int(bool(history)), sb, sl,
+                       VOXZIP_COMPACT_FILL if compaction == "fill" else VOXZIP_COMPACT_ORDERED)
+    d = desc.c_struct()
+    _check("voxzip_evict_ex", lib().voxzip_evict_ex(
+        ctypes.byref(d), int(layer_begin), int(layer_count), _ptr(k_cache), _ptr(v_cache), _ptr(score), _ptr(pos),
+        _ptr(len_), _ptr(budget), ctypes.byref(pol), _stream(stream)))
 
 
 def voxzip_get_status(stream=None) -> int:

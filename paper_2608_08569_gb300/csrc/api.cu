@@ -4,6 +4,7 @@
 
 #include "common.cuh"
 #include "embed.cuh"
+#include "evict_policy.cuh"
 
 namespace {
 
@@ -230,6 +231,27 @@ voxzip_status voxzip_evict(const voxzip_cache_desc *desc, int32_t layer_begin,
     return from_cuda(voxzip::launch_evict(*desc, layer_begin, layer_count, k_cache, v_cache, score, pos, len,
                                           budget, sink, recent_frac, status,
                                           reinterpret_cast<cudaStream_t>(stream)));
+}
+
+voxzip_status voxzip_evict_ex(const voxzip_cache_desc *desc, int32_t layer_begin,
+                              int32_t layer_count, void *k_cache, void *v_cache, float *score,
+                              int32_t *pos, int32_t *len, const int32_t *budget,
+                              const voxzip_evict_policy *policy, voxzip_stream_t stream) {
+    if (!desc_ok(desc) || policy == nullptr) return VOXZIP_EINVAL;
+    if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
+        return VOXZIP_EINVAL;
+    if (!k_cache || !v_cache || !score || !pos || !len || !budget) return VOXZIP_EINVAL;
+    const voxzip_evict_policy &p = *policy;
+    if (p.sink < 0 || !(p.recent_frac >= 0.f && p.recent_frac <= 1.f)) return VOXZIP_EINVAL;
+    if ((p.history != 0 && p.history != 1) || p.budget_stride_b < 0 || p.budget_stride_l < 0) return VOXZIP_EINVAL;
+    if (p.compaction != VOXZIP_COMPACT_ORDERED && p.compaction != VOXZIP_COMPACT_FILL) return VOXZIP_EINVAL;
+    if (!aligned16(k_cache) || !aligned16(v_cache)) return VOXZIP_EINVAL;
+    if ((int64_t)layer_count * desc->batch * desc->kv_heads > ((int64_t)1 << 31) - 1) return VOXZIP_EUNSUPPORTED;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    return from_cuda(voxzip::launch_evict_policy(*desc, layer_begin, layer_count, k_cache, v_cache, score, pos,
+                                                 len, budget, p, status, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 voxzip_status voxzip_get_status(uint32_t *bits, voxzip_stream_t stream) {

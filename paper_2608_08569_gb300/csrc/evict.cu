@@ -1,6 +1,10 @@
 // Budgeted eviction of VoxZip (Sec. 3.2.2, Eq. 7-9): keep T sinks, the M most recent rows and
 // the top-N history rows by decayed score, then compact K, V, score and pos in place.
+// Policy switches: the budget of a unit is read at budget[b * stride_b + layer * stride_l] (one
+// per sequence, or per layer); without history the recent window is budget - T rows (the
+// StreamingLLM baseline).
 //
+// evict_kernel (ordered compaction):
 // One CTA of 256 threads per unit (small enough that every unit of a launch is resident at once):
 //   select   MSB-first radix select (4 passes of 8 bits) over an order-preserving 32-bit image of
 //            the history scores gives the N-th best score. Only when that score is tied and not all
@@ -14,7 +18,15 @@
 //            later sub-chunk sit at slots >= its ranks, beyond every destination of an earlier one,
 //            so in-flight loads never see a store; and a barrier after all of a sub-chunk's loads
 //            have landed precedes its stores, so no row is overwritten before it is read.
+//
+// evict_fill_kernel (hole filling): sinks are the T lowest positions and the recent window the M
+// highest (radix selects over the positions), so the cache need not be in time order; the
+// history select is the same. Kept rows below the budget stay; the kept rows at slots >= budget
+// move, in ascending slot order, into the evicted slots below the budget, in ascending slot
+// order: at most n - budget rows move. Sources lie at or above the budget and destinations below
+// it, so no copy can read a row another one wrote.
 #include "common.cuh"
+#include "evict_policy.cuh"
 
 namespace voxzip {
 namespace {
@@ -31,8 +43,22 @@ struct EvictParams {
     const int32_t *budget;
     int32_t *status;
     int32_t B, L, Hkv, C, layer_begin, sink;
+    int32_t budget_stride_b, budget_stride_l, history;
     float recent_frac;
 };
+
+// The unit's budget and its split into T sinks, M recent rows and N history rows.
+struct Split {
+    int32_t bud, T, M, N;
+};
+__device__ __forceinline__ Split split_of(const EvictParams &p, const UnitIdx &ui) {
+    Split s;
+    s.bud = p.budget[(int64_t)ui.b * p.budget_stride_b + (int64_t)(p.layer_begin + ui.l_local) * p.budget_stride_l];
+    s.T = p.sink;
+    s.M = p.history ? (int32_t)floor((double)p.recent_frac * (double)s.bud) : s.bud - s.T;
+    s.N = s.bud - s.T - s.M;
+    return s;
+}
 
 __device__ __forceinline__ uint32_t score_key(float s) {  // monotone map of fp32 order to uint32 order
     const uint32_t b = __float_as_uint(s);
@@ -141,11 +167,9 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
     const int tid = threadIdx.x;
     const UnitIdx ui = unit_of(blockIdx.x, p.B, p.L, p.Hkv, p.layer_begin);
     const int32_t n = p.len[ui.cache_unit];
-    const int32_t bud = p.budget[ui.b];
-    const int32_t M = (int32_t)floor((double)p.recent_frac * (double)bud);
-    const int32_t T_ = p.sink;
-    const int32_t N = bud - T_ - M;
-    if (bud < 0 || N < 0) {
+    const Split sp = split_of(p, ui);
+    const int32_t bud = sp.bud, M = sp.M, T_ = sp.T, N = sp.N;
+    if (bud < 0 || N < 0 || M < 0) {
         if (tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_BUDGET);
         return;
     }
@@ -281,8 +305,147 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
 }
 
 template <typename T, int D>
-cudaError_t launch_t(const EvictParams &prm, int units, cudaStream_t stream) {
-    evict_kernel<T, D><<<units, kThreads, 0, stream>>>(prm);
+__global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictParams p) {
+    constexpr int kVecPerRow = D * (int)sizeof(T) / 16;
+    __shared__ int32_t holes[kSegment];
+    __shared__ int32_t movers[kSegment];
+    __shared__ unsigned hist[256];
+    __shared__ int warp_sums[32];
+    __shared__ RadixState shared_st;
+    __shared__ int resume_at;
+    const int tid = threadIdx.x;
+    const UnitIdx ui = unit_of(blockIdx.x, p.B, p.L, p.Hkv, p.layer_begin);
+    const int32_t n = p.len[ui.cache_unit];
+    const Split sp = split_of(p, ui);
+    const int32_t bud = sp.bud, M = sp.M, T_ = sp.T, N = sp.N;
+    if (bud < 0 || N < 0 || M < 0) {
+        if (tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_BUDGET);
+        return;
+    }
+    if (n <= bud) return;
+    if (n > p.C) {
+        if (tid == 0) raise_status(p.status, VOXZIP_DEV_CAPACITY);
+        return;
+    }
+    float *sc = p.score + ui.cache_unit * p.C;
+    int32_t *ps = p.pos + ui.cache_unit * p.C;
+    uint4 *kc = reinterpret_cast<uint4 *>(static_cast<T *>(p.k_cache) + ui.cache_unit * p.C * D);
+    uint4 *vc = reinterpret_cast<uint4 *>(static_cast<T *>(p.v_cache) + ui.cache_unit * p.C * D);
+
+    // Sinks: the T lowest positions (<= p_lo); recent window: the M highest (>= p_hi). Positions
+    // of a unit are unique, so each select cuts exactly.
+    auto pkey = [&](int j, bool &valid) {
+        valid = true;
+        return (uint32_t)ps[j];
+    };
+    uint32_t p_lo = 0u, p_hi = 0xffffffffu;
+    if (T_ > 0) {
+        RadixState st{0u, T_, 0};
+        for (int shift = 24; shift >= 0; shift -= 8) radix_pass<false>(shift, 0, n, pkey, st, hist, &shared_st);
+        p_lo = st.prefix;
+    }
+    if (M > 0) {
+        RadixState st{0u, M, 0};
+        for (int shift = 24; shift >= 0; shift -= 8) radix_pass<true>(shift, 0, n, pkey, st, hist, &shared_st);
+        p_hi = st.prefix;
+    }
+    auto middle = [&](uint32_t q) { return !(T_ > 0 && q <= p_lo) && !(M > 0 && q >= p_hi); };
+
+    // Eq. 9 over the rest, exactly as in the ordered eviction.
+    uint32_t thr = 0u, pos_thr = 0xffffffffu;
+    bool all_ties = true;
+    if (N > 0) {
+        RadixState st{0u, N, 0};
+        auto skey = [&](int j, bool &valid) {
+            valid = middle((uint32_t)ps[j]);
+            return score_key(sc[j]);
+        };
+        for (int shift = 24; shift >= 0; shift -= 8) radix_pass<true>(shift, 0, n, skey, st, hist, &shared_st);
+        thr = st.prefix;
+        all_ties = st.rem == st.bin;
+        if (!all_ties) {
+            RadixState sq{0u, st.rem, 0};
+            auto tkey = [&](int j, bool &valid) {
+                const uint32_t q = (uint32_t)ps[j];
+                valid = middle(q) && score_key(sc[j]) == thr;
+                return q;
+            };
+            for (int shift = 24; shift >= 0; shift -= 8)
+                radix_pass<false>(shift, 0, n, tkey, sq, hist, &shared_st);
+            pos_thr = sq.prefix;
+        }
+    }
+    auto kept = [&](int j) {
+        const uint32_t q = (uint32_t)ps[j];
+        if (!middle(q)) return true;
+        if (N == 0) return false;
+        const uint32_t k = score_key(sc[j]);
+        return k > thr || (k == thr && (all_ties || q <= pos_thr));
+    };
+
+    // Pair the evicted slots below the budget with the kept slots at or above it, in order, a
+    // segment of up to kSegment pairs at a time.
+    int hcur = 0, mcur = bud;
+    while (true) {
+        int nh = 0;
+        while (hcur < bud && nh + kThreads <= kSegment) {
+            const int j = hcur + tid;
+            const bool hole = j < bud && !kept(j);
+            int total;
+            const int r = scan_excl(hole ? 1 : 0, &total, warp_sums);
+            if (hole) holes[nh + r] = j;
+            nh += total;
+            hcur += kThreads;
+        }
+        if (nh == 0) break;
+        int nm = 0;
+        while (nm < nh && mcur < n) {
+            const int j = mcur + tid;
+            const bool mv = j < n && kept(j);
+            int total;
+            const int r = scan_excl(mv ? 1 : 0, &total, warp_sums);
+            if (mv && nm + r < nh) movers[nm + r] = j;
+            if (nm + total <= nh) {
+                nm += total;
+                mcur += kThreads;
+            } else {  // this step holds more movers than holes are left: resume after the last one taken
+                if (mv && nm + r == nh - 1) resume_at = j + 1;
+                __syncthreads();
+                mcur = resume_at;
+                nm = nh;
+                __syncthreads();
+            }
+        }
+        __syncthreads();
+        const int pairs = min(nh, nm);  // equal when positions are unique (then exactly `bud` rows are kept)
+        if (pairs < nh && tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_POSITIONS);
+        for (int v = tid; v < pairs * 2 * kVecPerRow; v += kThreads) {
+            const int row = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
+            uint4 *base = w < kVecPerRow ? kc : vc;
+            const int e = w % kVecPerRow;
+            base[(int64_t)holes[row] * kVecPerRow + e] = base[(int64_t)movers[row] * kVecPerRow + e];
+        }
+        for (int r = tid; r < pairs; r += kThreads) {
+            sc[holes[r]] = sc[movers[r]];
+            ps[holes[r]] = ps[movers[r]];
+        }
+        __syncthreads();
+        if (pairs < nh) break;
+    }
+    // Every kept row at or above the budget has found a hole; one left over means more than
+    // `bud` rows were kept (repeated positions).
+    int extra = 0;
+    for (int j = mcur + tid; j < n; j += kThreads) extra |= kept(j) ? 1 : 0;
+    if (__syncthreads_or(extra) && tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_POSITIONS);
+    if (tid == 0) p.len[ui.cache_unit] = bud;
+}
+
+template <typename T, int D>
+cudaError_t launch_t(const EvictParams &prm, int units, bool fill, cudaStream_t stream) {
+    if (fill)
+        evict_fill_kernel<T, D><<<units, kThreads, 0, stream>>>(prm);
+    else
+        evict_kernel<T, D><<<units, kThreads, 0, stream>>>(prm);
     return cudaGetLastError();
 }
 
@@ -292,16 +455,34 @@ cudaError_t launch_evict(const voxzip_cache_desc &d, int32_t layer_begin, int32_
                          void *k_cache, void *v_cache, float *score, int32_t *pos, int32_t *len,
                          const int32_t *budget, int32_t sink, float recent_frac, int32_t *status,
                          cudaStream_t stream) {
+    voxzip_evict_policy pol{};
+    pol.sink = sink;
+    pol.recent_frac = recent_frac;
+    pol.history = 1;
+    pol.budget_stride_b = 1;
+    pol.budget_stride_l = 0;
+    pol.compaction = VOXZIP_COMPACT_ORDERED;
+    return launch_evict_policy(d, layer_begin, layer_count, k_cache, v_cache, score, pos, len, budget, pol, status,
+                               stream);
+}
+
+cudaError_t launch_evict_policy(const voxzip_cache_desc &d, int32_t layer_begin, int32_t layer_count,
+                                void *k_cache, void *v_cache, float *score, int32_t *pos, int32_t *len,
+                                const int32_t *budget, const voxzip_evict_policy &pol, int32_t *status,
+                                cudaStream_t stream) {
     EvictParams prm;
     prm.k_cache = k_cache; prm.v_cache = v_cache; prm.score = score; prm.pos = pos; prm.len = len;
     prm.budget = budget; prm.status = status;
     prm.B = d.batch; prm.L = d.layers; prm.Hkv = d.kv_heads; prm.C = d.capacity;
-    prm.layer_begin = layer_begin; prm.sink = sink; prm.recent_frac = recent_frac;
+    prm.layer_begin = layer_begin; prm.sink = pol.sink; prm.recent_frac = pol.recent_frac;
+    prm.budget_stride_b = pol.budget_stride_b; prm.budget_stride_l = pol.budget_stride_l;
+    prm.history = pol.history;
     const int units = layer_count * d.batch * d.kv_heads;
-    const bool bf16 = d.dtype == VOXZIP_BF16;
+    const bool bf16 = d.dtype == VOXZIP_BF16, fill = pol.compaction == VOXZIP_COMPACT_FILL;
     if (d.head_dim == 128)
-        return bf16 ? launch_t<__nv_bfloat16, 128>(prm, units, stream) : launch_t<float, 128>(prm, units, stream);
-    return bf16 ? launch_t<__nv_bfloat16, 64>(prm, units, stream) : launch_t<float, 64>(prm, units, stream);
+        return bf16 ? launch_t<__nv_bfloat16, 128>(prm, units, fill, stream)
+                    : launch_t<float, 128>(prm, units, fill, stream);
+    return bf16 ? launch_t<__nv_bfloat16, 64>(prm, units, fill, stream) : launch_t<float, 64>(prm, units, fill, stream);
 }
 
 }  // namespace voxzip

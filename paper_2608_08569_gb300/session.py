@@ -13,15 +13,20 @@ from . import _native as N
 
 
 class Session:
+    """`budget` holds one budget per sequence, or per sequence and layer ([B][L]); `history` and
+    `compaction` select the eviction policy (see voxzip_evict_ex)."""
+
     def __init__(self, desc: N.CacheDesc, budget, gamma: float, *, sink: int = 4, recent_frac: float = 0.2,
-                 device="cuda", cache=None):
+                 history: bool = True, compaction: str = "ordered", device="cuda", cache=None):
         self.desc = desc
         self.device = torch.device(device)
         self.gamma = float(gamma)
         self.sink = int(sink)
         self.recent_frac = float(recent_frac)
-        self.budget_host = [int(b) for b in budget]
-        self.budget = torch.tensor(self.budget_host, dtype=torch.int32, device=self.device)
+        self.history = bool(history)
+        self.compaction = compaction
+        self.budget = torch.tensor(budget, dtype=torch.int32, device=self.device)
+        self.budget_host = [int(b) for b in self.budget.flatten().tolist()]
         self.cache = cache if cache is not None else N.allocate_cache(desc, self.device)
         self.n_max = 0
         self.workspace = None
@@ -56,7 +61,12 @@ class Session:
     def evict(self, *, layer_begin=0, layer_count=None, stream=None):
         c = self.cache
         lc = self.desc.layers if layer_count is None else layer_count
-        N.voxzip_evict(self.desc, layer_begin, lc, c["k"], c["v"], c["score"], c["pos"], c["len"], self.budget,
-                       sink=self.sink, recent_frac=self.recent_frac, stream=stream)
+        if self.history and self.compaction == "ordered" and self.budget.dim() == 1:
+            N.voxzip_evict(self.desc, layer_begin, lc, c["k"], c["v"], c["score"], c["pos"], c["len"], self.budget,
+                           sink=self.sink, recent_frac=self.recent_frac, stream=stream)
+        else:
+            N.voxzip_evict_ex(self.desc, layer_begin, lc, c["k"], c["v"], c["score"], c["pos"], c["len"],
+                              self.budget, sink=self.sink, recent_frac=self.recent_frac, history=self.history,
+                              compaction=self.compaction, stream=stream)
         if layer_begin + lc == self.desc.layers:
             self.n_max = min(self.n_max, max(self.budget_host))

@@ -64,13 +64,22 @@ def sample_units(w, k, seed=0):
     return sorted(pick)
 
 
-def gpu_run(w, inp, sample, steps=None, anchors=None):
-    """The whole path on the GPU through the C ABI; records the sampled units."""
+def unit_budget(w, policy, b, l):
+    """The budget of unit (b, l, .): per sequence, or per layer when the policy gives [B][L]."""
+    bl = (policy or {}).get("budget_bl")
+    return int(bl[b][l]) if bl is not None else int(w.budget[b])
+
+
+def gpu_run(w, inp, sample, steps=None, anchors=None, policy=None):
+    """The whole path on the GPU through the C ABI; records the sampled units. `policy` (optional)
+    holds history (bool), compaction ("ordered" / "fill") and budget_bl ([B][L] budgets)."""
     S = w.steps if steps is None else steps
     dev = inp["k_pre"].device
     B, L, Hq, H, D, G = w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.group
     desc = CacheDesc(B, L, Hq, H, D, w.capacity, w.dtype)
-    sess = Session(desc, w.budget, w.gamma, sink=w.sink, recent_frac=w.recent_frac, device=dev)
+    pol = policy or {}
+    sess = Session(desc, pol.get("budget_bl", w.budget), w.gamma, sink=w.sink, recent_frac=w.recent_frac,
+                   history=pol.get("history", True), compaction=pol.get("compaction", "ordered"), device=dev)
     sp = inp["spans"]
     i32 = lambda a: torch.as_tensor(np.asarray(a), dtype=torch.int32, device=dev)
     slot_map = torch.full((B, w.stride), -1, dtype=torch.int32, device=dev)
@@ -89,7 +98,7 @@ def gpu_run(w, inp, sample, steps=None, anchors=None):
                slot_map=slot_map.cpu().numpy())
     out = torch.empty(L, B, Hq, D, dtype=w.dtype, device=dev)
     outs, sb, lb, kp = [], [], [], []
-    maxbud = max(w.budget)
+    maxbud = max(sess.budget_host)
     for t in range(1, S + 1):
         sess.decode(inp["q"][t - 1], inp["kn"][t - 1], inp["vn"][t - 1], inp["new_pos"][t - 1], out)
         outs.append(out[li, bi].view(len(sample), H, G, D)[ar, hi].clone())
@@ -119,7 +128,7 @@ def _anchor_unit(anchors, w, spans, b, l, h):
     return f(anchors[0]), f(anchors[1])
 
 
-def oracle_units(w, inp, sample, steps=None, anchors=None, workers=None):
+def oracle_units(w, inp, sample, steps=None, anchors=None, workers=None, policy=None):
     """run_unit of the oracle for every sampled unit, in parallel threads (ctypes drops the GIL)."""
     S = w.steps if steps is None else steps
     orc = oracle.default()
@@ -128,16 +137,18 @@ def oracle_units(w, inp, sample, steps=None, anchors=None, workers=None):
         u = W.unit_inputs(w, inp["spans"], inp["k_pre"], inp["v_pre"], inp["q"], inp["kn"], inp["vn"],
                           inp["new_pos"], b, l, h, steps=S)
         ak, av = _anchor_unit(anchors, w, inp["spans"], b, l, h)
-        args.append((u, ak, av, b))
+        args.append((u, ak, av, b, l))
+    pol = policy or {}
 
     def one(a):
-        u, ak, av, b = a
+        u, ak, av, b, l = a
         return orc.run_unit(u["xk"], u["xv"], u["in_len"], u["audio_begin"], u["audio_len"], u["span_start"],
                             u["span_end"], u["span_groups"], q=u["q"], k_new=u["k_new"], v_new=u["v_new"],
                             new_pos=u["new_pos"], gamma=w.gamma, scale=1.0 / math.sqrt(w.head_dim),
-                            interval=w.interval, budget=w.budget[b], sink=w.sink, recent_frac=w.recent_frac,
-                            capacity=w.capacity, anchor_k=ak, anchor_v=av,
-                            cache_is_bf16=w.dtype == torch.bfloat16)
+                            interval=w.interval, budget=unit_budget(w, policy, b, l), sink=w.sink,
+                            recent_frac=w.recent_frac, capacity=w.capacity, anchor_k=ak, anchor_v=av,
+                            cache_is_bf16=w.dtype == torch.bfloat16, history=pol.get("history", True),
+                            fill=pol.get("compaction", "ordered") == "fill")
 
     with cf.ThreadPoolExecutor(max_workers=workers or os.cpu_count() or 4) as ex:
         return list(ex.map(one, args))
@@ -164,21 +175,25 @@ def check_stage1(w, inp, rec, sample, anchors=None):
             np.testing.assert_array_equal(rec["slot_map"][b, :u["in_len"]], r["slot_map"])
 
 
-def _nth_score(scores, n, T, M, N):
-    cand = np.sort(scores[T:n - M])[::-1]
+def _nth_score(scores, n, T, M, N, pos=None):
+    """The N-th best history score; the history lies between the sinks and the recent window in
+    slot order, or in position order when `pos` is given (hole-filling caches)."""
+    mid = scores[T:n - M] if pos is None else scores[np.argsort(pos[:n], kind="stable")][T:n - M]
+    cand = np.sort(mid)[::-1]
     return cand[N - 1] if N >= 1 else math.inf
 
 
-def check_units(w, rec, orc_results, sample, steps=None):
+def check_units(w, rec, orc_results, sample, steps=None, policy=None):
     """Lockstep comparison; returns the list of units that legitimately diverged at a near-tie."""
+    pol = policy or {}
     S = w.steps if steps is None else steps
     tol = out_tol(w)
     assert rec["status"] == 0, f"device status bits {rec['status']:#x}"
     diverged = []
     stats = dict(max_out_err=0.0, max_score_rel=0.0, evictions=0)
     for i, ((b, l, h), o) in enumerate(zip(sample, orc_results)):
-        bud = w.budget[b]
-        M = math.floor(float(np.float32(w.recent_frac)) * bud)
+        bud = unit_budget(w, policy, b, l)
+        M = math.floor(float(np.float32(w.recent_frac)) * bud) if pol.get("history", True) else bud - w.sink
         N = bud - w.sink - M
         ev = 0
         gone = False
@@ -199,7 +214,8 @@ def check_units(w, rec, orc_results, sample, steps=None):
                                    f"{(np.abs(gs - os_) / np.maximum(np.abs(os_), 1e-30)).max():.3g}")
             m = min(n, bud)
             if not np.array_equal(rec["kept_pos"][ev, i, :m], o["kept_pos"][ev, :m]):
-                thr = _nth_score(os_, n, w.sink, M, N)
+                thr = _nth_score(os_, n, w.sink, M, N,
+                                 pos=o["pos_before"][ev] if pol.get("compaction") == "fill" else None)
                 assert o["margin"][ev] <= SCORE_RTOL * thr + SCORE_ATOL, (
                     f"unit {(b, l, h)} eviction {ev}: kept sets differ with margin {o['margin'][ev]:.3g} "
                     f"(threshold score {thr:.3g})")
