@@ -52,6 +52,8 @@ def parse_args():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-units", type=int, default=0, help="units in the oracle sample (0: one per core)")
+    p.add_argument("--compaction", choices=["ordered", "fill"], default="ordered",
+                   help="eviction compaction: ordered (Eq. 7-8, default) or hole filling")
     p.add_argument("--part", choices=["path", "embed"], default="path",
                    help="path: the KV-compression path (default); embed: embedding-level stage 1")
     return p.parse_args()
@@ -197,10 +199,11 @@ def decode_bytes(w, n_after):
 
 
 def evict_bytes(w, n_before, moved_rows):
-    """Bytes an ordered in-place eviction must move (Eq. 7-8): each unit over budget reads its
-    scores and positions once for the selection (8 B per slot), and every kept row that changes
-    slot (all kept rows after the first evicted slot) is read and written with its K, V, score and
-    position. moved_rows[u] is counted from the positions before and after the eviction."""
+    """Bytes an eviction must move (Eq. 7-8): each unit over budget reads its scores and positions
+    once for the selection (8 B per slot), and every kept row that changes slot is read and
+    written with its K, V, score and position. That is every kept row after the first evicted slot
+    for the ordered compaction, and at most n - budget rows for hole filling. moved_rows[u] is
+    counted from the positions before and after the eviction."""
     es = 2 if w.dtype == torch.bfloat16 else 4
     row = 2 * w.head_dim * es + 8
     return int(8 * int(n_before.sum()) + 2 * row * int(moved_rows.sum()))
@@ -209,7 +212,7 @@ def evict_bytes(w, n_before, moved_rows):
 # ----------------------------------------------------------------------------- GPU arm
 
 class Runner:
-    def __init__(self, w, device):
+    def __init__(self, w, device, compaction="ordered"):
         from paper_2608_08569_gb300 import CacheDesc
         from paper_2608_08569_gb300 import workloads as W
         from paper_2608_08569_gb300.session import Session
@@ -222,7 +225,8 @@ class Runner:
         self.k_pre, self.v_pre = W.make_prefill(w, device)
         self.q, self.kn, self.vn, self.npos = W.make_steps(w, device)
         self.desc = CacheDesc(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.capacity, w.dtype)
-        self.sess = Session(self.desc, w.budget, w.gamma, sink=w.sink, recent_frac=w.recent_frac, device=device)
+        self.sess = Session(self.desc, w.budget, w.gamma, sink=w.sink, recent_frac=w.recent_frac,
+                            compaction=compaction, device=device)
         self.out = torch.empty(w.steps, w.layers, w.batch, w.q_heads, w.head_dim, dtype=w.dtype, device=device)
 
     def request(self, timers=None, lengths=None, evict_timers=None, moved=None):
@@ -265,8 +269,8 @@ class Runner:
 
 
 def moved_rows(pos_before, n_before, pos_after, n_after):
-    """(lengths before, rows that changed slot) per unit of one eviction: a unit that shrank keeps
-    its rows up to the first slot whose position changed and moves every kept row after it."""
+    """(lengths before, rows that changed slot) per unit of one eviction: the slots below the new
+    length whose position changed received a row (positions of a unit are unique)."""
     C = pos_before.shape[-1]
     pb = pos_before.reshape(-1, C)
     pa = pos_after.reshape(-1, C)
@@ -274,9 +278,8 @@ def moved_rows(pos_before, n_before, pos_after, n_after):
     na = n_after.reshape(-1).long()
     idx = torch.arange(C, device=pb.device)
     differs = (pb != pa) & (idx[None, :] < na[:, None])
-    first = torch.where(differs.any(1), differs.float().argmax(1), na)
     shrank = na < nb
-    moved = torch.where(shrank, na - first, torch.zeros_like(na))
+    moved = torch.where(shrank, differs.sum(1), torch.zeros_like(na))
     return nb[shrank].cpu().numpy(), moved.cpu().numpy()
 
 
@@ -285,7 +288,7 @@ def gpu_arm(args, rank, world, local):
     w = W.CONFIGS[args.workload]
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
-    r = Runner(w, dev)
+    r = Runner(w, dev, compaction=args.compaction)
     for _ in range(args.warmup):
         r.request()
     torch.cuda.synchronize()
@@ -347,12 +350,15 @@ def gpu_arm(args, rank, world, local):
     ev_ms = sum(a.elapsed_time(b) for a, b in ev_timers)
     if ev_timers and ev_ms > 0:
         ev_ach = ev_bytes * args.steps / (ev_ms / 1000.0) / 1e9
-        etr = profiled_traffic_ratio("evict_kernel_stress.md", ["evict.cu", "common.cuh"])
+        etr = profiled_traffic_ratio("evict_kernel_stress.md", ["evict.cu", "common.cuh"]) \
+            if args.compaction == "ordered" else None
         roofline_evict = {"bound": "hbm", "achieved": round(ev_ach, 1), "peak": peak, "unit": "GB/s",
                           "frac": round(ev_ach / peak, 4),
                           "traffic": None if etr is None or w.name != "stress" else
                           int(etr * ev_bytes / max(1, len(moved))),
-                          "kernel": "evict_kernel (top-N select + ordered in-place compaction)",
+                          "kernel": "evict_kernel (top-N select + ordered in-place compaction)"
+                          if args.compaction == "ordered" else
+                          "evict_fill_kernel (top-N select + hole-filling compaction)",
                           "avg_launch_us": round(1000.0 * ev_ms / len(ev_timers), 2),
                           "alg_bytes_per_launch": int(ev_bytes / max(1, len(moved))),
                           "evict_share_of_step": round(ev_ms / ms, 4)}
@@ -372,13 +378,14 @@ def gpu_arm(args, rank, world, local):
                    "q_heads": w.q_heads, "kv_heads": w.kv_heads, "head_dim": w.head_dim,
                    "prompt_tokens": list(sorted(set(w.in_len))), "budget": list(sorted(set(w.budget))),
                    "gamma": w.gamma, "decode_steps_per_request": w.steps, "evict_interval": w.interval,
+                   "compaction": args.compaction,
                    "parallelism": f"replicas x{world} (independent units, no collective)",
                    "l2": "inputs larger than L2 (decode reads ~0.9-7 GB per launch, L2 is 129 MB)"},
         "roofline": roofline, "roofline_evict": roofline_evict, "gpu_launches": gpu_launches, "clocks": clocks,
         "e2e": e2e,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        result["cpu_baseline"] = cpu_sample(w, args.cpu_units)
+        result["cpu_baseline"] = cpu_sample(w, args.cpu_units, compaction=args.compaction)
     return result
 
 
@@ -459,7 +466,7 @@ def sample_units(w, k):
     return [all_units[i] for i in sorted(idx)]
 
 
-def cpu_sample(w, n_units=0, inputs=None):
+def cpu_sample(w, n_units=0, inputs=None, compaction="ordered"):
     """Times the oracle on a bounded sample: `n_units` units (one per thread), each through the
     whole request; the whole-workload time is the sample's wall time x units / sampled units."""
     import oracle
@@ -478,7 +485,7 @@ def cpu_sample(w, n_units=0, inputs=None):
                             u["span_end"], u["span_groups"], q=u["q"], k_new=u["k_new"], v_new=u["v_new"],
                             new_pos=u["new_pos"], gamma=w.gamma, scale=1.0 / math.sqrt(w.head_dim),
                             interval=w.interval, budget=w.budget[b], sink=w.sink, recent_frac=w.recent_frac,
-                            capacity=w.capacity, cache_is_bf16=w.dtype == torch.bfloat16)
+                            capacity=w.capacity, cache_is_bf16=w.dtype == torch.bfloat16, fill=compaction == "fill")
 
     args = [(u, b) for u, (b, l, h) in zip(inputs, units)]
     used = min(threads, len(args))
@@ -501,11 +508,11 @@ def reference_arm(args, rank, world):
         return None
     inputs = None
     for _ in range(args.warmup):
-        _, inputs = cpu_sample(w, args.cpu_units, inputs)
+        _, inputs = cpu_sample(w, args.cpu_units, inputs, args.compaction)
     vals, last = [], None
     t0 = time.perf_counter()
     for _ in range(args.steps):
-        last, inputs = cpu_sample(w, args.cpu_units, inputs)
+        last, inputs = cpu_sample(w, args.cpu_units, inputs, args.compaction)
         vals.append(last["value"])
     wall = time.perf_counter() - t0
     value = statistics.mean(vals)

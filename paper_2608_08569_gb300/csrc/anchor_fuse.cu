@@ -16,11 +16,25 @@
 //   fuse_wide   embedding level, any width that is a whole number of 16-byte vectors: one warp per
 //               output row of a sequence, the same arithmetic.
 // Output slots cover the kept tokens of the prompt in order, each a contiguous source range.
+#include <algorithm>
+
 #include "common.cuh"
 #include "embed.cuh"
 
 namespace voxzip {
 namespace {
+
+// SMs of the current device (looked up once per device).
+int sm_count() {
+    static int cached[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 148;
+    if (cached[dev] == 0) {
+        int n = 0;
+        cached[dev] = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0 ? n : 148;
+    }
+    return cached[dev];
+}
 
 constexpr int kScanThreads = 512;
 constexpr int kMapThreads = 256;
@@ -238,7 +252,9 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
     const int32_t *src = ws.slot_src + (int64_t)b * stride;
     const int32_t *send = ws.slot_end + (int64_t)b * stride;
     const int32_t *anc = ws.slot_anchor + (int64_t)b * stride;
-    const int slot0 = (blockIdx.x * kFuseWarps + warp) * kSlotsPerWarp * kRowsPerWarp;
+    constexpr int kSlotsPerPass = kFuseWarps * kSlotsPerWarp * kRowsPerWarp;
+    for (int slot0 = (blockIdx.x * kFuseWarps + warp) * kSlotsPerWarp * kRowsPerWarp; slot0 < out_len;
+         slot0 += gridDim.x * kSlotsPerPass)
     for (int k = 0; k < kSlotsPerWarp; ++k) {
         const int s = slot0 + k * kRowsPerWarp + sub;
         if (s >= out_len) break;
@@ -283,8 +299,12 @@ cudaError_t launch_fuse_rows(const voxzip_cache_desc &d, int32_t stride, int32_t
     constexpr int kRowsPerWarp = 32 / (D / 4);
     const int slots_per_block = kFuseWarps * kSlotsPerWarp * kRowsPerWarp;
     const int64_t units = (int64_t)d.batch * d.layers * d.kv_heads;
-    dim3 grid((unsigned)((stride + slots_per_block - 1) / slots_per_block), (unsigned)units);
-    if (grid.x == 0) grid.x = 1;
+    // A grid-stride loop over each unit's output slots: about six CTAs per SM in all, never more
+    // than the prompt stride needs (stage 1 leaves far fewer slots than prompt tokens).
+    const int64_t per_unit = (sm_count() * 6 + units - 1) / units;
+    dim3 grid((unsigned)std::max<int64_t>(1, std::min<int64_t>((stride + slots_per_block - 1) / slots_per_block,
+                                                               per_unit)),
+              (unsigned)units);
     fuse_rows_kernel<T, D><<<grid, kFuseWarps * 32, 0, stream>>>(
         d.batch, d.layers, d.kv_heads, d.capacity, stride, anchor_stride, (const T *)kp, (const T *)vp,
         (const T *)ak, (const T *)av, ws, (T *)kc, (T *)vc, score, pos, len);
@@ -363,10 +383,26 @@ fuse_wide_kernel(int32_t C, int32_t stride, int32_t D, int32_t text_stride, cons
             for (int h = 0; h < 2; ++h)
 #pragma unroll
                 for (int e = 0; e < kElems; ++e) acc[h][e] = 0.f;
-            for (int32_t r = r0; r < r1; ++r) {
-                const T *row = in + (int64_t)r * D;
-                const uint4 x0 = *reinterpret_cast<const uint4 *>(row + v0 * kElems);
-                const uint4 x1 = two ? *reinterpret_cast<const uint4 *>(row + (v0 + 32) * kElems) : x0;
+            const uint4 *col = reinterpret_cast<const uint4 *>(in) + v0;   // vector v0 of row 0
+            const int64_t rstride = vecs;                                    // vectors per row
+            int32_t r = r0;
+            // Four source rows' loads in flight, then their sums in token order.
+            for (; r + 4 <= r1; r += 4) {
+                uint4 x[4][2];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    x[i][0] = __ldcs(col + (int64_t)(r + i) * rstride);
+                    x[i][1] = two ? __ldcs(col + (int64_t)(r + i) * rstride + 32) : x[i][0];
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    accumulate16<T>(acc[0], x[i][0]);
+                    accumulate16<T>(acc[1], x[i][1]);
+                }
+            }
+            for (; r < r1; ++r) {
+                const uint4 x0 = __ldcs(col + (int64_t)r * rstride);
+                const uint4 x1 = two ? __ldcs(col + (int64_t)r * rstride + 32) : x0;
                 accumulate16<T>(acc[0], x0);
                 accumulate16<T>(acc[1], x1);
             }
@@ -464,7 +500,10 @@ cudaError_t launch_embed_fuse(int32_t B, int32_t D, int32_t C, bool bf16, const 
                                        in_len, audio_begin, audio_len, span_off, span_start, span_end, span_groups,
                                        ws, slot_map, status, stream);
     if (err != cudaSuccess) return err;
-    dim3 grid((unsigned)((stride + kWideWarps - 1) / kWideWarps), (unsigned)B);
+    // A grid-stride loop over the output rows; about five CTAs of 8 warps per SM in all (the
+    // output has far fewer rows than the prompt stride the slot plan is sized for).
+    const int per_seq = (sm_count() * 5 + B - 1) / B;
+    dim3 grid((unsigned)max(1, min((stride + kWideWarps - 1) / kWideWarps, per_seq)), (unsigned)B);
     if (bf16)
         fuse_wide_kernel<__nv_bfloat16><<<grid, kWideWarps * 32, 0, stream>>>(
             C, stride, D, text_stride, (const __nv_bfloat16 *)e_in, (const __nv_bfloat16 *)e_text, ws,
