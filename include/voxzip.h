@@ -301,6 +301,69 @@ voxzip_status voxzip_evict_ex(const voxzip_cache_desc *desc, int32_t layer_begin
                               const voxzip_evict_policy *policy, voxzip_stream_t stream);
 
 /*
+ * Paged cache (for serving many turns: memory follows the live cache, not a fixed capacity).
+ *
+ * K and V rows live in pools of pages of VOXZIP_PAGE_TOKENS rows. Slot s of unit u is row
+ * (s % 64) of page page_table[u][s / 64]; scores, positions and lengths stay dense as in the
+ * cache layout above (8 bytes per slot). Free pages are a device-side stack, so every call of the
+ * decode loop runs without a host round trip and can be captured in a CUDA graph:
+ *   - voxzip_paged_init gives unit u page u for slot 0 and stacks the rest as free;
+ *   - voxzip_anchor_fuse_paged returns each unit's pages and takes the ones its stage-1 rows need;
+ *   - voxzip_decode_step_paged takes a page when an append fills the unit's last one;
+ *   - voxzip_evict_paged returns the pages beyond the budget.
+ * After every call a unit of length n holds the pages of slots [0, n] (the next append's slot
+ * included) when the pool allowed it. A decode whose slot has no page, or a stage 1 the pool
+ * cannot hold, sets VOXZIP_DEV_CAPACITY and skips the unit. Which free page a unit receives depends
+ * on the order in which units ran, so it is not deterministic.
+ */
+#define VOXZIP_PAGE_TOKENS 64
+
+typedef struct {
+    void *k_pool;        /* [pages][64][D] in the descriptor's dtype, 16-byte aligned */
+    void *v_pool;        /* [pages][64][D] */
+    int32_t *page_table; /* [B][L][Hkv][max_pages] device int32: page of slots [64 p, 64 p + 64), -1 none */
+    int32_t *free_pages; /* [pages] device int32: stack of free page indices */
+    int32_t *free_count; /* device int32: stack entries in use */
+    int32_t pages;       /* pool size; at least B * L * Hkv */
+    int32_t max_pages;   /* pages per unit; the descriptor's capacity must be 64 * max_pages */
+} voxzip_paged_cache;
+
+/* Empty every unit (len = 0, page u of the pool for its slot 0) and stack the other pages. */
+voxzip_status voxzip_paged_init(const voxzip_cache_desc *desc, const voxzip_paged_cache *paged,
+                                int32_t *len, voxzip_stream_t stream);
+
+/* voxzip_anchor_fuse into a paged cache (same arguments and results; K/V rows go to the pages). */
+voxzip_status voxzip_anchor_fuse_paged(const voxzip_cache_desc *desc, const voxzip_paged_cache *paged,
+                                       const void *k_prefill, const void *v_prefill,
+                                       int32_t prefill_stride, const int32_t *in_len,
+                                       const int32_t *audio_begin, const int32_t *audio_len,
+                                       const int32_t *span_off, int32_t num_spans,
+                                       const int32_t *span_start, const int32_t *span_end,
+                                       const int32_t *span_groups, const void *anchor_k,
+                                       const void *anchor_v, int32_t anchor_stride, float *score,
+                                       int32_t *pos, int32_t *len, int32_t *slot_map, void *workspace,
+                                       size_t workspace_bytes, voxzip_stream_t stream);
+
+/* Bytes of workspace voxzip_anchor_fuse_paged needs (0 if the arguments are invalid). */
+size_t voxzip_anchor_fuse_paged_workspace_size(const voxzip_cache_desc *desc, int32_t prefill_stride,
+                                               int32_t num_spans);
+
+/* voxzip_decode_step on a paged cache (bf16, head_dim 64 or 128, group <= 16; else
+   VOXZIP_EUNSUPPORTED). */
+voxzip_status voxzip_decode_step_paged(const voxzip_cache_desc *desc, const voxzip_paged_cache *paged,
+                                       int32_t layer_begin, int32_t layer_count, const void *q,
+                                       const void *k_new, const void *v_new, const int32_t *new_pos,
+                                       float *score, int32_t *pos, int32_t *len, float gamma,
+                                       float sm_scale, int32_t max_len, void *out,
+                                       voxzip_stream_t stream);
+
+/* voxzip_evict_ex on a paged cache; the pages beyond the new length's are returned. */
+voxzip_status voxzip_evict_paged(const voxzip_cache_desc *desc, const voxzip_paged_cache *paged,
+                                 int32_t layer_begin, int32_t layer_count, float *score, int32_t *pos,
+                                 int32_t *len, const int32_t *budget, const voxzip_evict_policy *policy,
+                                 voxzip_stream_t stream);
+
+/*
  * Waits for `stream`, then returns the device status word of the current device in *bits
  * (VOXZIP_DEV_* flags accumulated by earlier calls) and clears it.
  */

@@ -79,6 +79,14 @@ class _EvictPolicy(ctypes.Structure):
                 ("compaction", ctypes.c_int32)]
 
 
+class _Paged(ctypes.Structure):
+    _fields_ = [("k_pool", ctypes.c_void_p), ("v_pool", ctypes.c_void_p), ("page_table", ctypes.c_void_p),
+                ("free_pages", ctypes.c_void_p), ("free_count", ctypes.c_void_p), ("pages", ctypes.c_int32),
+                ("max_pages", ctypes.c_int32)]
+
+
+PAGE_TOKENS = 64
+
 _lock = threading.Lock()
 _lib = None
 _vp = ctypes.c_void_p
@@ -111,6 +119,16 @@ def lib() -> ctypes.CDLL:
             L.voxzip_get_status.argtypes = [ctypes.POINTER(ctypes.c_uint32), _vp]
             L.voxzip_evict_ex.argtypes = [_DP, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp,
                                           ctypes.POINTER(_EvictPolicy), _vp]
+            _PP = ctypes.POINTER(_Paged)
+            L.voxzip_paged_init.argtypes = [_DP, _PP, _vp, _vp]
+            L.voxzip_anchor_fuse_paged.argtypes = [_DP, _PP, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp,
+                                                   _vp, _vp, _i32, _vp, _vp, _vp, _vp, _vp, _sz, _vp]
+            L.voxzip_anchor_fuse_paged_workspace_size.argtypes = [_DP, _i32, _i32]
+            L.voxzip_anchor_fuse_paged_workspace_size.restype = _sz
+            L.voxzip_decode_step_paged.argtypes = [_DP, _PP, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _f32,
+                                                   _f32, _i32, _vp, _vp]
+            L.voxzip_evict_paged.argtypes = [_DP, _PP, _i32, _i32, _vp, _vp, _vp, _vp, ctypes.POINTER(_EvictPolicy),
+                                             _vp]
             L.voxzip_segments_to_spans.argtypes = [_i32, _vp, _vp, _vp, _vp, _f64, _i32, _i32, _f64, _vp, _vp, _vp,
                                                    _vp, _vp]
             L.voxzip_embed_fuse.argtypes = [_EP, _vp, _i32, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _i32,
@@ -121,7 +139,8 @@ def lib() -> ctypes.CDLL:
             L.voxzip_status_string.restype = ctypes.c_char_p
             L.voxzip_version.restype = _i32
             for f in (L.voxzip_anchor_fuse, L.voxzip_decode_step, L.voxzip_evict, L.voxzip_get_status,
-                      L.voxzip_segments_to_spans, L.voxzip_embed_fuse, L.voxzip_evict_ex):
+                      L.voxzip_segments_to_spans, L.voxzip_embed_fuse, L.voxzip_evict_ex, L.voxzip_paged_init,
+                      L.voxzip_anchor_fuse_paged, L.voxzip_decode_step_paged, L.voxzip_evict_paged):
                 f.restype = _i32
             _lib = L
     return _lib
@@ -171,6 +190,128 @@ def allocate_cache(desc: CacheDesc, device="cuda"):
                 score=torch.zeros(cs, dtype=torch.float32, device=device),
                 pos=torch.zeros(cs, dtype=torch.int32, device=device),
                 len=torch.zeros(cs[:3], dtype=torch.int32, device=device))
+
+
+def allocate_paged_cache(desc: CacheDesc, pages: int, device="cuda", stream=None):
+    """A paged cache: K and V page pools of `pages` pages of 64 rows, the page table and the free
+    stack, and the dense per-slot state (score, pos, len). desc.capacity (a multiple of 64) bounds
+    one unit. The cache starts empty (voxzip_paged_init)."""
+    if desc.capacity % PAGE_TOKENS:
+        raise ValueError("a paged cache's capacity must be a multiple of 64")
+    cs = (desc.batch, desc.layers, desc.kv_heads, desc.capacity)
+    mp = desc.capacity // PAGE_TOKENS
+    pc = dict(k_pool=torch.zeros(pages, PAGE_TOKENS, desc.head_dim, dtype=desc.dtype, device=device),
+              v_pool=torch.zeros(pages, PAGE_TOKENS, desc.head_dim, dtype=desc.dtype, device=device),
+              page_table=torch.full(cs[:3] + (mp,), -1, dtype=torch.int32, device=device),
+              free_pages=torch.zeros(pages, dtype=torch.int32, device=device),
+              free_count=torch.zeros(1, dtype=torch.int32, device=device),
+              score=torch.zeros(cs, dtype=torch.float32, device=device),
+              pos=torch.zeros(cs, dtype=torch.int32, device=device),
+              len=torch.zeros(cs[:3], dtype=torch.int32, device=device), pages=int(pages), max_pages=mp)
+    voxzip_paged_init(desc, pc, stream=stream)
+    return pc
+
+
+def _paged_struct(desc: CacheDesc, pc) -> _Paged:
+    mp = desc.capacity // PAGE_TOKENS
+    _need(pc["k_pool"], "k_pool", desc.dtype, (pc["pages"], PAGE_TOKENS, desc.head_dim))
+    _need(pc["v_pool"], "v_pool", desc.dtype, (pc["pages"], PAGE_TOKENS, desc.head_dim))
+    _need(pc["page_table"], "page_table", torch.int32, (desc.batch, desc.layers, desc.kv_heads, mp))
+    _need(pc["free_pages"], "free_pages", torch.int32, (pc["pages"],))
+    _need(pc["free_count"], "free_count", torch.int32, (1,))
+    return _Paged(pc["k_pool"].data_ptr(), pc["v_pool"].data_ptr(), pc["page_table"].data_ptr(),
+                  pc["free_pages"].data_ptr(), pc["free_count"].data_ptr(), int(pc["pages"]), mp)
+
+
+def _check_dense_state(desc: CacheDesc, score, pos, len_) -> None:
+    cs = (desc.batch, desc.layers, desc.kv_heads, desc.capacity)
+    _need(score, "score", torch.float32, cs)
+    _need(pos, "pos", torch.int32, cs)
+    _need(len_, "len", torch.int32, cs[:3])
+
+
+def voxzip_paged_init(desc: CacheDesc, pc, stream=None) -> None:
+    """Empties every unit of a paged cache (page u for unit u's slot 0, the rest free)."""
+    d, ps = desc.c_struct(), _paged_struct(desc, pc)
+    _need(pc["len"], "len", torch.int32, (desc.batch, desc.layers, desc.kv_heads))
+    _check("voxzip_paged_init", lib().voxzip_paged_init(ctypes.byref(d), ctypes.byref(ps), _ptr(pc["len"]),
+                                                        _stream(stream)))
+
+
+def paged_pages_in_use(pc) -> int:
+    """Pages held by units (synchronises with the device)."""
+    return int(pc["pages"]) - int(pc["free_count"].item())
+
+
+def voxzip_anchor_fuse_paged(desc: CacheDesc, pc, k_prefill, v_prefill, in_len, audio_begin, audio_len, span_off,
+                             span_start, span_end, span_groups, *, slot_map=None, anchor_k=None, anchor_v=None,
+                             workspace=None, stream=None) -> None:
+    """Stage 1 (Sec. 3.2.1) into a paged cache: each unit returns its pages and takes the ones its
+    stage-1 rows need."""
+    B, L, H, D = desc.batch, desc.layers, desc.kv_heads, desc.head_dim
+    stride = k_prefill.shape[3]
+    _need(k_prefill, "k_prefill", desc.dtype, (B, L, H, stride, D))
+    _need(v_prefill, "v_prefill", desc.dtype, (B, L, H, stride, D))
+    for name, t in (("in_len", in_len), ("audio_begin", audio_begin), ("audio_len", audio_len)):
+        _need(t, name, torch.int32, (B,))
+    _need(span_off, "span_off", torch.int32, (B + 1,))
+    num_spans = span_start.numel()
+    _check_dense_state(desc, pc["score"], pc["pos"], pc["len"])
+    if slot_map is not None:
+        _need(slot_map, "slot_map", torch.int32, (B, stride))
+    anchor_stride = 0
+    if anchor_k is not None or anchor_v is not None:
+        anchor_stride = anchor_k.shape[3]
+        _need(anchor_k, "anchor_k", desc.dtype, (B, L, H, anchor_stride, D))
+        _need(anchor_v, "anchor_v", desc.dtype, (B, L, H, anchor_stride, D))
+    d, ps = desc.c_struct(), _paged_struct(desc, pc)
+    need = int(lib().voxzip_anchor_fuse_paged_workspace_size(ctypes.byref(d), int(stride), int(num_spans)))
+    if workspace is None or workspace.numel() < need:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=k_prefill.device)
+    _check("voxzip_anchor_fuse_paged", lib().voxzip_anchor_fuse_paged(
+        ctypes.byref(d), ctypes.byref(ps), _ptr(k_prefill), _ptr(v_prefill), int(stride), _ptr(in_len),
+        _ptr(audio_begin), _ptr(audio_len), _ptr(span_off), int(num_spans), _ptr(span_start), _ptr(span_end),
+        _ptr(span_groups), _ptr(anchor_k), _ptr(anchor_v), int(anchor_stride), _ptr(pc["score"]), _ptr(pc["pos"]),
+        _ptr(pc["len"]), _ptr(slot_map), _ptr(workspace), int(workspace.numel()), _stream(stream)))
+
+
+def voxzip_decode_step_paged(desc: CacheDesc, pc, layer_begin: int, layer_count: int, q, k_new, v_new, new_pos,
+                             gamma: float, out, *, sm_scale: float = 0.0, max_len: int = 0, stream=None) -> None:
+    """One decode step (Eq. 1, Eq. 2, Eq. 6) on a paged cache."""
+    B, Hq, H, D = desc.batch, desc.q_heads, desc.kv_heads, desc.head_dim
+    _need(q, "q", desc.dtype, (layer_count, B, Hq, D))
+    _need(k_new, "k_new", desc.dtype, (layer_count, B, H, D))
+    _need(v_new, "v_new", desc.dtype, (layer_count, B, H, D))
+    _need(out, "out", desc.dtype, (layer_count, B, Hq, D))
+    _need(new_pos, "new_pos", torch.int32, (B,))
+    _check_dense_state(desc, pc["score"], pc["pos"], pc["len"])
+    d, ps = desc.c_struct(), _paged_struct(desc, pc)
+    _check("voxzip_decode_step_paged", lib().voxzip_decode_step_paged(
+        ctypes.byref(d), ctypes.byref(ps), int(layer_begin), int(layer_count), _ptr(q), _ptr(k_new), _ptr(v_new),
+        _ptr(new_pos), _ptr(pc["score"]), _ptr(pc["pos"]), _ptr(pc["len"]), float(gamma), float(sm_scale),
+        int(max_len), _ptr(out), _stream(stream)))
+
+
+def voxzip_evict_paged(desc: CacheDesc, pc, layer_begin: int, layer_count: int, budget, *, sink: int = 4,
+                       recent_frac: float = 0.2, history: bool = True, compaction: str = "ordered",
+                       stream=None) -> None:
+    """Eviction (Eq. 7-9, under a policy as voxzip_evict_ex) on a paged cache; the pages beyond the
+    new length go back to the pool."""
+    _check_dense_state(desc, pc["score"], pc["pos"], pc["len"])
+    if budget.dim() == 1:
+        _need(budget, "budget", torch.int32, (desc.batch,))
+        sb, sl = 1, 0
+    else:
+        _need(budget, "budget", torch.int32, (desc.batch, desc.layers))
+        sb, sl = desc.layers, 1
+    if compaction not in ("ordered", "fill"):
+        raise ValueError("compaction must be 'ordered' or 'fill'")
+    pol = _EvictPolicy(int(sink), float(recent_frac), int(bool(history)), sb, sl,
+                       VOXZIP_COMPACT_FILL if compaction == "fill" else VOXZIP_COMPACT_ORDERED)
+    d, ps = desc.c_struct(), _paged_struct(desc, pc)
+    _check("voxzip_evict_paged", lib().voxzip_evict_paged(
+        ctypes.byref(d), ctypes.byref(ps), int(layer_begin), int(layer_count), _ptr(pc["score"]), _ptr(pc["pos"]),
+        _ptr(pc["len"]), _ptr(budget), ctypes.byref(pol), _stream(stream)))
 
 
 def voxzip_anchor_fuse_workspace_size(desc: CacheDesc, prefill_stride: int, num_spans: int) -> int:

@@ -20,6 +20,7 @@
 
 #include "common.cuh"
 #include "embed.cuh"
+#include "paged.cuh"
 
 namespace voxzip {
 namespace {
@@ -230,24 +231,26 @@ slot_map_kernel(int32_t stride, bool keep_bg, const int32_t *__restrict__ in_len
     }
 }
 
-template <typename T, int D>
+// kPaged: k_cache / v_cache are page pools and output slot s goes to the row the page table gives.
+template <typename T, int D, bool kPaged>
 __global__ void __launch_bounds__(kFuseWarps * 32)
 fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, int32_t anchor_stride,
                  const T *__restrict__ k_prefill, const T *__restrict__ v_prefill,
                  const T *__restrict__ anchor_k, const T *__restrict__ anchor_v, FuseWorkspace ws,
                  T *__restrict__ k_cache, T *__restrict__ v_cache, float *__restrict__ score,
-                 int32_t *__restrict__ pos, int32_t *__restrict__ len) {
+                 int32_t *__restrict__ pos, int32_t *__restrict__ len, PageView pv) {
     constexpr int kLanesPerRow = D / 4;          // each lane owns 4 consecutive elements
     constexpr int kRowsPerWarp = 32 / kLanesPerRow;
     const int u = blockIdx.y;                    // cache unit (b, l, h)
     const int b = u / (L * Hkv);
-    const int32_t out_len = ws.seq_len[b];
+    int32_t out_len = ws.seq_len[b];
+    if (kPaged && pv.table[(int64_t)u * pv.max_pages] < 0) out_len = -1;  // the pool could not hold it
     if (blockIdx.x == 0 && threadIdx.x == 0) len[u] = out_len < 0 ? 0 : out_len;
     if (out_len < 0) return;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / kLanesPerRow, e = (lane % kLanesPerRow) * 4;
     const int64_t in_base = (int64_t)u * stride * D;
-    const int64_t out_base = (int64_t)u * C * D;
+    const int64_t out_base = kPaged ? 0 : (int64_t)u * C * D;
     const int64_t anc_base = (int64_t)u * anchor_stride * D;
     const int32_t *src = ws.slot_src + (int64_t)b * stride;
     const int32_t *send = ws.slot_end + (int64_t)b * stride;
@@ -282,8 +285,9 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
             sv.x = __fadd_rn(sv.x, av.x); sv.y = __fadd_rn(sv.y, av.y);
             sv.z = __fadd_rn(sv.z, av.z); sv.w = __fadd_rn(sv.w, av.w);
         }
-        store4(k_cache + out_base + (int64_t)s * D + e, sk);
-        store4(v_cache + out_base + (int64_t)s * D + e, sv);
+        const int64_t orow = kPaged ? paged_row(pv, u, s) : s;
+        store4(k_cache + out_base + orow * D + e, sk);
+        store4(v_cache + out_base + orow * D + e, sv);
         if (e == 0) {
             pos[(int64_t)u * C + s] = r0;
             score[(int64_t)u * C + s] = 0.f;
@@ -291,11 +295,11 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
     }
 }
 
-template <typename T, int D>
+template <typename T, int D, bool kPaged = false>
 cudaError_t launch_fuse_rows(const voxzip_cache_desc &d, int32_t stride, int32_t anchor_stride,
                              const void *kp, const void *vp, const void *ak, const void *av,
                              const FuseWorkspace &ws, void *kc, void *vc, float *score, int32_t *pos,
-                             int32_t *len, cudaStream_t stream) {
+                             int32_t *len, cudaStream_t stream, PageView pv = PageView{nullptr, nullptr, nullptr, 0}) {
     constexpr int kRowsPerWarp = 32 / (D / 4);
     const int slots_per_block = kFuseWarps * kSlotsPerWarp * kRowsPerWarp;
     const int64_t units = (int64_t)d.batch * d.layers * d.kv_heads;
@@ -305,9 +309,9 @@ cudaError_t launch_fuse_rows(const voxzip_cache_desc &d, int32_t stride, int32_t
     dim3 grid((unsigned)std::max<int64_t>(1, std::min<int64_t>((stride + slots_per_block - 1) / slots_per_block,
                                                                per_unit)),
               (unsigned)units);
-    fuse_rows_kernel<T, D><<<grid, kFuseWarps * 32, 0, stream>>>(
+    fuse_rows_kernel<T, D, kPaged><<<grid, kFuseWarps * 32, 0, stream>>>(
         d.batch, d.layers, d.kv_heads, d.capacity, stride, anchor_stride, (const T *)kp, (const T *)vp,
-        (const T *)ak, (const T *)av, ws, (T *)kc, (T *)vc, score, pos, len);
+        (const T *)ak, (const T *)av, ws, (T *)kc, (T *)vc, score, pos, len, pv);
     return cudaGetLastError();
 }
 
@@ -428,6 +432,35 @@ fuse_wide_kernel(int32_t C, int32_t stride, int32_t D, int32_t text_stride, cons
     }
 }
 
+// Paged stage 1, step 1: every unit of the launch returns all its pages (one warp per unit).
+__global__ void __launch_bounds__(256) page_release_kernel(int64_t units, PageView pv) {
+    const int64_t u = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+    if (u < units) return_pages_warp(pv, u, 0, pv.max_pages);
+}
+
+// Step 2: each unit takes the pages of slots [0, n] for its stage-1 length n (all or none; none
+// leaves page 0 missing, which the fusion and later calls read as "skipped").
+__global__ void __launch_bounds__(256) page_take_kernel(int64_t units, int32_t per_seq, FuseWorkspace ws, PageView pv,
+                                                        int32_t *status) {
+    const int64_t u = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (u >= units) return;
+    const int32_t n = max(0, ws.seq_len[u / per_seq]);
+    const int32_t need = min(n / kPageTokens + 1, pv.max_pages);  // a full unit needs no page for slot n
+    int32_t top = 0;
+    if (lane == 0) {
+        top = atomicSub(pv.free_count, need);
+        if (top < need) {  // not enough: give them back (whatever other units did meanwhile)
+            atomicAdd(pv.free_count, need);
+            raise_status(status, VOXZIP_DEV_CAPACITY);
+            top = -1;
+        }
+    }
+    top = __shfl_sync(0xffffffffu, top, 0);
+    if (top < 0) return;
+    for (int32_t p = lane; p < need; p += 32) pv.table[u * pv.max_pages + p] = pv.free_pages[top - need + p];
+}
+
 // span_scan then slot_map: the slot, source range and anchor row of every output row.
 cudaError_t launch_slot_plan(int32_t B, int32_t capacity, int32_t stride, int32_t num_spans, int32_t anchor_stride,
                              bool has_anchor, bool keep_bg, const int32_t *in_len, const int32_t *audio_begin,
@@ -478,6 +511,67 @@ cudaError_t launch_anchor_fuse(const voxzip_cache_desc &d, const void *k_prefill
                                                        stream)
                 : launch_fuse_rows<float, 64>(d, prefill_stride, anchor_stride, k_prefill, v_prefill, anchor_k,
                                               anchor_v, ws, k_cache, v_cache, score, pos, len, stream);
+}
+
+size_t anchor_fuse_paged_workspace_bytes(const voxzip_cache_desc &d, int32_t prefill_stride, int32_t num_spans) {
+    return carve(d, prefill_stride, num_spans, nullptr, nullptr);
+}
+
+cudaError_t launch_anchor_fuse_paged(const voxzip_cache_desc &d, const voxzip_paged_cache &pc, const void *k_prefill,
+                                     const void *v_prefill, int32_t prefill_stride, const int32_t *in_len,
+                                     const int32_t *audio_begin, const int32_t *audio_len, const int32_t *span_off,
+                                     int32_t num_spans, const int32_t *span_start, const int32_t *span_end,
+                                     const int32_t *span_groups, const void *anchor_k, const void *anchor_v,
+                                     int32_t anchor_stride, float *score, int32_t *pos, int32_t *len,
+                                     int32_t *slot_map, void *workspace, int32_t *status, cudaStream_t stream) {
+    FuseWorkspace ws;
+    carve(d, prefill_stride, num_spans, static_cast<char *>(workspace), &ws);
+    const PageView pv{pc.page_table, pc.free_pages, pc.free_count, pc.max_pages};
+    const int64_t units = (int64_t)d.batch * d.layers * d.kv_heads;
+    const unsigned blocks = (unsigned)((units + 7) / 8);
+    page_release_kernel<<<blocks, 256, 0, stream>>>(units, pv);
+    cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    err = launch_slot_plan(d.batch, d.capacity, prefill_stride, num_spans, anchor_stride, anchor_k != nullptr, true,
+                           in_len, audio_begin, audio_len, span_off, span_start, span_end, span_groups, ws, slot_map,
+                           status, stream);
+    if (err != cudaSuccess) return err;
+    page_take_kernel<<<blocks, 256, 0, stream>>>(units, d.layers * d.kv_heads, ws, pv, status);
+    err = cudaGetLastError();
+    if (err != cudaSuccess) return err;
+    const bool bf16 = d.dtype == VOXZIP_BF16;
+    void *kc = pc.k_pool, *vc = pc.v_pool;
+    if (d.head_dim == 128)
+        return bf16 ? launch_fuse_rows<__nv_bfloat16, 128, true>(d, prefill_stride, anchor_stride, k_prefill, v_prefill,
+                                                                  anchor_k, anchor_v, ws, kc, vc, score, pos, len,
+                                                                  stream, pv)
+                    : launch_fuse_rows<float, 128, true>(d, prefill_stride, anchor_stride, k_prefill, v_prefill,
+                                                         anchor_k, anchor_v, ws, kc, vc, score, pos, len, stream, pv);
+    return bf16 ? launch_fuse_rows<__nv_bfloat16, 64, true>(d, prefill_stride, anchor_stride, k_prefill, v_prefill,
+                                                             anchor_k, anchor_v, ws, kc, vc, score, pos, len, stream,
+                                                             pv)
+                : launch_fuse_rows<float, 64, true>(d, prefill_stride, anchor_stride, k_prefill, v_prefill, anchor_k,
+                                                    anchor_v, ws, kc, vc, score, pos, len, stream, pv);
+}
+
+// Empty units: page u holds unit u's slot 0, the other pages are stacked free, lengths are 0.
+__global__ void paged_init_kernel(int64_t units, int32_t max_pages, int32_t pages, int32_t *table,
+                                  int32_t *free_pages, int32_t *free_count, int32_t *len) {
+    const int64_t stride = (int64_t)gridDim.x * blockDim.x;
+    const int64_t first = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    for (int64_t i = first; i < units * max_pages; i += stride)
+        table[i] = i % max_pages == 0 ? (int32_t)(i / max_pages) : -1;
+    for (int64_t j = first; j < pages - units; j += stride) free_pages[j] = (int32_t)(units + j);
+    for (int64_t u = first; u < units; u += stride) len[u] = 0;
+    if (first == 0) *free_count = (int32_t)(pages - units);
+}
+
+cudaError_t launch_paged_init(const voxzip_cache_desc &d, const voxzip_paged_cache &pc, int32_t *len,
+                              cudaStream_t stream) {
+    const int64_t units = (int64_t)d.batch * d.layers * d.kv_heads;
+    paged_init_kernel<<<sm_count() * 4, 256, 0, stream>>>(units, pc.max_pages, pc.pages, pc.page_table,
+                                                          pc.free_pages, pc.free_count, len);
+    return cudaGetLastError();
 }
 
 size_t embed_fuse_workspace_bytes(int32_t batch, int32_t stride, int32_t num_spans) {

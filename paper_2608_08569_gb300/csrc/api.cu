@@ -5,6 +5,7 @@
 #include "common.cuh"
 #include "embed.cuh"
 #include "evict_policy.cuh"
+#include "paged.cuh"
 
 namespace {
 
@@ -103,6 +104,110 @@ voxzip_status voxzip_anchor_fuse(const voxzip_cache_desc *desc, const void *k_pr
         *desc, k_prefill, v_prefill, prefill_stride, in_len, audio_begin, audio_len, span_off, num_spans,
         span_start, span_end, span_groups, anchor_k, anchor_v, anchor_stride, k_cache, v_cache, score, pos, len,
         slot_map, workspace, status, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+namespace {
+bool paged_ok(const voxzip_cache_desc *d, const voxzip_paged_cache *pc) {
+    if (!desc_ok(d) || pc == nullptr) return false;
+    if (!pc->k_pool || !pc->v_pool || !pc->page_table || !pc->free_pages || !pc->free_count) return false;
+    if (!aligned16(pc->k_pool) || !aligned16(pc->v_pool)) return false;
+    const int64_t units = (int64_t)d->batch * d->layers * d->kv_heads;
+    if (pc->max_pages < 1 || (int64_t)pc->max_pages * VOXZIP_PAGE_TOKENS != d->capacity) return false;
+    if (pc->pages < units || (int64_t)pc->pages * VOXZIP_PAGE_TOKENS > INT32_MAX) return false;
+    return true;
+}
+
+bool policy_ok(const voxzip_evict_policy &p) {
+    if (p.sink < 0 || !(p.recent_frac >= 0.f && p.recent_frac <= 1.f)) return false;
+    if ((p.history != 0 && p.history != 1) || p.budget_stride_b < 0 || p.budget_stride_l < 0) return false;
+    return p.compaction == VOXZIP_COMPACT_ORDERED || p.compaction == VOXZIP_COMPACT_FILL;
+}
+}  // namespace
+
+voxzip_status voxzip_paged_init(const voxzip_cache_desc *desc, const voxzip_paged_cache *paged, int32_t *len,
+                                voxzip_stream_t stream) {
+    if (!paged_ok(desc, paged) || !len) return VOXZIP_EINVAL;
+    return from_cuda(voxzip::launch_paged_init(*desc, *paged, len, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+size_t voxzip_anchor_fuse_paged_workspace_size(const voxzip_cache_desc *desc, int32_t prefill_stride,
+                                               int32_t num_spans) {
+    if (!desc_ok(desc) || prefill_stride < 1 || num_spans < 0) return 0;
+    return voxzip::anchor_fuse_paged_workspace_bytes(*desc, prefill_stride, num_spans);
+}
+
+voxzip_status voxzip_anchor_fuse_paged(const voxzip_cache_desc *desc, const voxzip_paged_cache *paged,
+                                       const void *k_prefill, const void *v_prefill,
+                                       int32_t prefill_stride, const int32_t *in_len,
+                                       const int32_t *audio_begin, const int32_t *audio_len,
+                                       const int32_t *span_off, int32_t num_spans,
+                                       const int32_t *span_start, const int32_t *span_end,
+                                       const int32_t *span_groups, const void *anchor_k,
+                                       const void *anchor_v, int32_t anchor_stride, float *score,
+                                       int32_t *pos, int32_t *len, int32_t *slot_map, void *workspace,
+                                       size_t workspace_bytes, voxzip_stream_t stream) {
+    if (!paged_ok(desc, paged) || prefill_stride < 1 || num_spans < 0) return VOXZIP_EINVAL;
+    if (!k_prefill || !v_prefill || !in_len || !audio_begin || !audio_len || !span_off || !score || !pos || !len ||
+        !workspace)
+        return VOXZIP_EINVAL;
+    if (num_spans > 0 && (!span_start || !span_end || !span_groups)) return VOXZIP_EINVAL;
+    if ((anchor_k == nullptr) != (anchor_v == nullptr)) return VOXZIP_EINVAL;
+    if (anchor_k && anchor_stride < 1) return VOXZIP_EINVAL;
+    if (!aligned16(k_prefill) || !aligned16(v_prefill) || (anchor_k && (!aligned16(anchor_k) || !aligned16(anchor_v))))
+        return VOXZIP_EINVAL;
+    if ((reinterpret_cast<uintptr_t>(workspace) & 255u) != 0) return VOXZIP_EINVAL;
+    if (workspace_bytes < voxzip::anchor_fuse_paged_workspace_bytes(*desc, prefill_stride, num_spans))
+        return VOXZIP_EINVAL;
+    if ((int64_t)desc->batch * desc->layers * desc->kv_heads > kMaxGridY || desc->batch > kMaxGridY)
+        return VOXZIP_EUNSUPPORTED;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    return from_cuda(voxzip::launch_anchor_fuse_paged(
+        *desc, *paged, k_prefill, v_prefill, prefill_stride, in_len, audio_begin, audio_len, span_off, num_spans,
+        span_start, span_end, span_groups, anchor_k, anchor_v, anchor_stride, score, pos, len, slot_map, workspace,
+        status, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+voxzip_status voxzip_decode_step_paged(const voxzip_cache_desc *desc, const voxzip_paged_cache *paged,
+                                       int32_t layer_begin, int32_t layer_count, const void *q,
+                                       const void *k_new, const void *v_new, const int32_t *new_pos,
+                                       float *score, int32_t *pos, int32_t *len, float gamma,
+                                       float sm_scale, int32_t max_len, void *out,
+                                       voxzip_stream_t stream) {
+    if (!paged_ok(desc, paged)) return VOXZIP_EINVAL;
+    if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
+        return VOXZIP_EINVAL;
+    if (!q || !k_new || !v_new || !new_pos || !score || !pos || !len || !out) return VOXZIP_EINVAL;
+    if (!(gamma > 0.f && gamma <= 1.f) || isnan(sm_scale) || isinf(sm_scale)) return VOXZIP_EINVAL;
+    if (!aligned16(q) || !aligned16(k_new) || !aligned16(v_new) || !aligned16(out)) return VOXZIP_EINVAL;
+    if (!voxzip::decode_mma_paged_supported(*desc)) return VOXZIP_EUNSUPPORTED;
+    if ((int64_t)layer_count * desc->batch * desc->kv_heads > kMaxGridY) return VOXZIP_EUNSUPPORTED;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    bool unsupported = false;
+    cudaError_t e = voxzip::launch_decode_mma_paged(*desc, *paged, layer_begin, layer_count, q, k_new, v_new, new_pos,
+                                                    score, pos, len, gamma, sm_scale, max_len, out, status,
+                                                    reinterpret_cast<cudaStream_t>(stream), &unsupported);
+    if (unsupported) return VOXZIP_EUNSUPPORTED;
+    return from_cuda(e);
+}
+
+voxzip_status voxzip_evict_paged(const voxzip_cache_desc *desc, const voxzip_paged_cache *paged,
+                                 int32_t layer_begin, int32_t layer_count, float *score, int32_t *pos,
+                                 int32_t *len, const int32_t *budget, const voxzip_evict_policy *policy,
+                                 voxzip_stream_t stream) {
+    if (!paged_ok(desc, paged) || policy == nullptr || !policy_ok(*policy)) return VOXZIP_EINVAL;
+    if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
+        return VOXZIP_EINVAL;
+    if (!score || !pos || !len || !budget) return VOXZIP_EINVAL;
+    if ((int64_t)layer_count * desc->batch * desc->kv_heads > ((int64_t)1 << 31) - 1) return VOXZIP_EUNSUPPORTED;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    return from_cuda(voxzip::launch_evict_paged(*desc, *paged, layer_begin, layer_count, score, pos, len, budget,
+                                                *policy, status, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 voxzip_status voxzip_segments_to_spans(int32_t n, const double *t_start, const double *t_end,

@@ -16,9 +16,12 @@
 // G x D outputs from all CTAs' partials. (Exchanging the statistics between the two phases instead
 // makes every CTA wait twice for the slowest one of its cluster, which measured slower.)
 // The appended row is patched into its tile in shared memory, so no load waits for its store.
+// Paged caches (kPaged): a CTA's range is whole 64-token pages, each tile is loaded from the pool
+// row its page-table entry gives, and the CTA that completes a page takes the next one.
 #include <cooperative_groups.h>
 
 #include "common.cuh"
+#include "paged.cuh"
 #include "ptx.cuh"
 #include "tmap.cuh"
 
@@ -54,6 +57,7 @@ constexpr int kBoxBytes = kTile * kBoxCols * 2;
 constexpr uint32_t kWaitLimit = 1u << 24;
 constexpr size_t kMaxSmem = 227 * 1024;
 constexpr int kMaxCluster = 16;
+static_assert(kTile == kPageTokens, "a paged cache's page is one tile of the ring");
 
 struct MmaParams {
     const __nv_bfloat16 *q, *k_new, *v_new;
@@ -65,6 +69,7 @@ struct MmaParams {
     int32_t *status;
     int32_t B, L, Hq, Hkv, G, C, layer_begin, chunk_cap, n_hint;
     float gamma, scale_log2;
+    PageView pv;  // paged instantiations: the pools are k_cache / v_cache
 };
 
 template <int D, int NT, int kStages>
@@ -82,8 +87,9 @@ struct Layout {
     static constexpr int kStatOff = kPbufOff + kPbufBytes;     // m_w, z_w [warps][kGP]; m_cta, z_cta [kGP]; fac [S][kGP]
     static constexpr int kStatFloats = (2 * kConsumerWarps + 2 + kMaxCluster) * kGP;
     static constexpr int kLgOff = kStatOff + kStatFloats * 4;  // logits / p [chunk_cap][kGP] fp32, then old scores
-    static size_t bytes(int chunk_cap) {
-        return 1024 + (size_t)kLgOff + (size_t)chunk_cap * kGP * 4 + (size_t)chunk_cap * 4;
+    static size_t bytes(int chunk_cap) {  // + the pool row of each tile (paged)
+        return 1024 + (size_t)kLgOff + (size_t)chunk_cap * kGP * 4 + (size_t)chunk_cap * 4 +
+               (size_t)(chunk_cap / kTile + 1) * 4;
     }
 };
 
@@ -92,7 +98,8 @@ __device__ __forceinline__ uint32_t swz(int row, int chunk) {  // byte offset in
 }
 
 // kCluster: launched in clusters of S > 1 CTAs (else one CTA holds the whole unit).
-template <int D, int NT, int kStages, bool kCluster>
+// kPaged: K/V rows live in page pools (see paged.cuh).
+template <int D, int NT, int kStages, bool kCluster, bool kPaged>
 __global__ void __launch_bounds__(kThreads)
 decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant__ CUtensorMap tmv,
                   const MmaParams p) {
@@ -123,13 +130,14 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     float *fac = z_cta + GP;                                   // [S][GP]: 2^(m_r - m) / Z; 0 for padding heads
     float *lg = reinterpret_cast<float *>(smem + Lay::kLgOff);
     float *s_old = lg + (size_t)p.chunk_cap * GP;               // [chunk_cap] scores before the step
+    int32_t *tile_rows = reinterpret_cast<int32_t *>(s_old + p.chunk_cap);  // [tiles] pool row (paged)
 
     const UnitIdx ui = unit_of(blockIdx.y, p.B, p.L, p.Hkv, p.layer_begin);
     const int64_t act_row = (int64_t)ui.l_local * p.B + ui.b;
     const int64_t row_base = ui.cache_unit * p.C;
     // While this unit's length is read, pull the first tiles of the range the launch's length hint
     // predicts into L2 (exact when the unit is as long as the hint; otherwise a few wasted KB).
-    if (warp == kConsumerWarps && lane == 0) {
+    if (!kPaged && warp == kConsumerWarps && lane == 0) {
         const int est_j0 = rank * ((p.n_hint + S - 1) / S);
         const int rows = min(kStages * kTile, p.C - est_j0);
         if (rows > 0) ptx::prefetch_l2(p.k_cache + (row_base + est_j0) * D, (uint32_t)rows * D * 2);
@@ -160,7 +168,15 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         if (rank == 0 && tid == 0) raise_status(p.status, VOXZIP_DEV_CAPACITY);
         return;
     }
-    const int chunk = (n + S - 1) / S;
+    int32_t page_new = 0;  // paged: page of the appended row (slot n - 1)
+    if constexpr (kPaged) {
+        page_new = p.pv.table[ui.cache_unit * p.pv.max_pages + (n_old >> 6)];
+        if (page_new < 0) {  // the pool had no page for it: the same decision in every CTA
+            if (rank == 0 && tid == 0) raise_status(p.status, VOXZIP_DEV_CAPACITY);
+            return;
+        }
+    }
+    const int chunk = kPaged ? ((n + S - 1) / S + kTile - 1) / kTile * kTile : (n + S - 1) / S;
     if (chunk > p.chunk_cap) {
         if (rank == 0 && tid == 0) raise_status(p.status, VOXZIP_DEV_LEN_HINT);
         return;
@@ -182,7 +198,8 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         const int64_t src = (act_row * p.Hkv + ui.h) * D + lane * 8;
         kn4 = *reinterpret_cast<const uint4 *>(p.k_new + src);
         vn4 = *reinterpret_cast<const uint4 *>(p.v_new + src);
-        const int64_t dst = (row_base + n - 1) * D + lane * 8;
+        const int64_t dst = (kPaged ? (int64_t)page_new * kPageTokens + (n_old & (kPageTokens - 1)) : row_base + n - 1) * D +
+                            lane * 8;
         *reinterpret_cast<uint4 *>(p.k_cache + dst) = kn4;
         *reinterpret_cast<uint4 *>(p.v_cache + dst) = vn4;
         if (lane == 0) p.pos[row_base + n - 1] = p.new_pos[ui.b];
@@ -207,6 +224,11 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     bool ok = true;
     if (warp == kConsumerWarps) {
         // ------------------------------------------------------------- producer
+        if constexpr (kPaged) {  // the pool row of every tile of the range (j0 is page-aligned)
+            const int32_t *trow = p.pv.table + ui.cache_unit * p.pv.max_pages + j0 / kTile;
+            for (int t = lane; t < ntiles; t += 32) tile_rows[t] = trow[t] * kTile;
+            __syncwarp();
+        }
         if (lane == 0 && ntiles > 0) {
             ptx::prefetch_tmap(&tmk);
             ptx::prefetch_tmap(&tmv);
@@ -219,7 +241,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                 ptx::mbar_arrive_expect_tx(&full[s], Lay::kStageBytes);
                 const bool is_k = i < ntiles;
                 const int tile = is_k ? i : i - ntiles;
-                const int32_t y = (int32_t)(row_base + j0 + tile * kTile);
+                const int32_t y = kPaged ? tile_rows[tile] : (int32_t)(row_base + j0 + tile * kTile);
                 uint8_t *dst = stages + s * Lay::kStageBytes;
 #pragma unroll
                 for (int h = 0; h < kHalves; ++h)
@@ -529,7 +551,15 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         }
     }
     if (clustered) cluster.sync();  // no CTA leaves while others may still read its shared memory
-    if (rank == 0 && tid == 0) p.len[ui.cache_unit] = n;
+    if (rank == 0 && tid == 0) {
+        p.len[ui.cache_unit] = n;
+        if constexpr (kPaged) {  // the next append starts a page: take one now
+            if ((n & (kPageTokens - 1)) == 0 && (n >> 6) < p.pv.max_pages) {
+                int32_t *entry = p.pv.table + ui.cache_unit * p.pv.max_pages + (n >> 6);
+                if (*entry < 0) *entry = take_page(p.pv);
+            }
+        }
+    }
 }
 
 // ---------------------------------------------------------------- host side
@@ -560,15 +590,17 @@ auto dispatch(int D, int NT, int NS, F &&f) {
 using KernelFn = void (*)(CUtensorMap, CUtensorMap, MmaParams);
 
 template <typename K>
-KernelFn kernel_for(int S) {
-    return S > 1 ? decode_mma_kernel<K::D, K::NT, K::NS, true> : decode_mma_kernel<K::D, K::NT, K::NS, false>;
+KernelFn kernel_for(int S, bool paged = false) {
+    if (paged)
+        return S > 1 ? decode_mma_kernel<K::D, K::NT, K::NS, true, true> : decode_mma_kernel<K::D, K::NT, K::NS, false, true>;
+    return S > 1 ? decode_mma_kernel<K::D, K::NT, K::NS, true, false> : decode_mma_kernel<K::D, K::NT, K::NS, false, false>;
 }
 
 template <typename K>
 bool configure() {  // kernel attributes are per function; set once per process
     static bool done = false;
     if (!done) {
-        for (KernelFn kern : {kernel_for<K>(1), kernel_for<K>(2)})
+        for (KernelFn kern : {kernel_for<K>(1), kernel_for<K>(2), kernel_for<K>(1, true), kernel_for<K>(2, true)})
             if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kMaxSmem) != cudaSuccess ||
                 cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
                 return false;
@@ -602,8 +634,8 @@ int max_active_clusters(int S, size_t smem) {
 
 template <typename K>
 cudaError_t launch_t(const CUtensorMap &tmk, const CUtensorMap &tmv, const MmaParams &prm, int S, int units,
-                     cudaStream_t stream) {
-    const KernelFn kern = kernel_for<K>(S);
+                     cudaStream_t stream, bool paged) {
+    const KernelFn kern = kernel_for<K>(S, paged);
     if (!configure<K>()) return cudaErrorInvalidValue;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)S, (unsigned)units, 1);
@@ -637,7 +669,7 @@ constexpr PlanModel kPlanModel{VOXZIP_DECODE_CTA_FIXED_US, VOXZIP_DECODE_CLUSTER
 // in turn; a unit costs a CTA's fixed latency (more with a cluster exchange) plus its tokens at one
 // CTA's streaming rate, which grows with the ring stages in flight until the CTAs resident on an SM
 // share its bandwidth; and no launch beats the GPU's streaming rate.
-Plan plan(int D, int NT, int units, int nmax, const PlanModel &md = kPlanModel) {
+Plan plan(int D, int NT, int units, int nmax, bool paged = false, const PlanModel &md = kPlanModel) {
     Plan best{0, 3, 0};
     double best_cost = 0.0;
     int sms = 148;
@@ -649,7 +681,7 @@ Plan plan(int D, int NT, int units, int nmax, const PlanModel &md = kPlanModel) 
     for (int S = 1; S <= kMaxCluster; S <<= 1) {
         int cap = (nmax + S - 1) / S;
         if (S > 1 && cap < kTile / 2) break;
-        cap = (cap + 15) / 16 * 16;
+        cap = paged ? (cap + kTile - 1) / kTile * kTile : (cap + 15) / 16 * 16;  // paged: whole pages per CTA
         for (int ns : kRingDepths) {
             const size_t sm = dispatch(D, NT, ns, [&](auto k) {
                 using K = decltype(k);
@@ -682,18 +714,24 @@ bool decode_mma_supported(const voxzip_cache_desc &d) {
            tensor_map_encoder() != nullptr;
 }
 
-cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, int32_t layer_count, const void *q,
-                              const void *k_new, const void *v_new, const int32_t *new_pos, void *k_cache,
-                              void *v_cache, float *score, int32_t *pos, int32_t *len, float gamma, float sm_scale,
-                              int32_t max_len, void *out, int32_t *status, cudaStream_t stream, bool *unsupported) {
+namespace {
+
+// The dense and the paged launch: K/V rows are [rows][D] at k_base / v_base (the cache, or the
+// page pools), pv.table is null for the dense layout.
+cudaError_t launch_impl(const voxzip_cache_desc &d, void *k_base, void *v_base, int64_t rows, const PageView &pv,
+                        int32_t layer_begin, int32_t layer_count, const void *q, const void *k_new, const void *v_new,
+                        const int32_t *new_pos, float *score, int32_t *pos, int32_t *len, float gamma, float sm_scale,
+                        int32_t max_len, void *out, int32_t *status, cudaStream_t stream, bool *unsupported) {
     *unsupported = false;
+    const bool paged = pv.table != nullptr;
     const int G = d.q_heads / d.kv_heads;
     const int NT = G <= 8 ? 1 : 2;
     const int units = layer_count * d.batch * d.kv_heads;
     const int nmax = (max_len > 0 && max_len < d.capacity) ? max_len : d.capacity;
-    // Plans are cached per (head dim, group tiles, units, length bucket of one tile).
+    // Plans are cached per (head dim, group tiles, units, length bucket of one tile, layout).
     struct Entry {
         int D, NT, units, bucket;
+        bool paged;
         Plan p;
     };
     thread_local Entry cache[16];
@@ -701,32 +739,33 @@ cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, i
     const int bucket = (nmax + kTile - 1) / kTile;
     Plan pl{0, 0, 0};
     for (const Entry &e : cache)
-        if (e.p.S != 0 && e.D == d.head_dim && e.NT == NT && e.units == units && e.bucket == bucket) pl = e.p;
+        if (e.p.S != 0 && e.D == d.head_dim && e.NT == NT && e.units == units && e.bucket == bucket &&
+            e.paged == paged)
+            pl = e.p;
     if (pl.S == 0) {
-        pl = plan(d.head_dim, NT, units, bucket * kTile);
+        pl = plan(d.head_dim, NT, units, bucket * kTile, paged);
         if (pl.S == 0) {
             *unsupported = true;
             return cudaSuccess;
         }
-        cache[cache_next] = Entry{d.head_dim, NT, units, bucket, pl};
+        cache[cache_next] = Entry{d.head_dim, NT, units, bucket, paged, pl};
         cache_next = (cache_next + 1) % 16;
     }
     const int S = pl.S;
     const int chunk_cap = pl.chunk_cap;
-    const int64_t rows = (int64_t)d.batch * d.layers * d.kv_heads * d.capacity;
     thread_local void *cached_k = nullptr, *cached_v = nullptr;
     thread_local int64_t cached_rows = 0;
     thread_local int cached_d = 0;
     thread_local CUtensorMap tmk, tmv;
-    if (cached_k != k_cache || cached_v != v_cache || cached_rows != rows || cached_d != d.head_dim) {
-        if (!make_cache_map(&tmk, k_cache, rows, d.head_dim, kTile) ||
-            !make_cache_map(&tmv, v_cache, rows, d.head_dim, kTile)) {
+    if (cached_k != k_base || cached_v != v_base || cached_rows != rows || cached_d != d.head_dim) {
+        if (!make_cache_map(&tmk, k_base, rows, d.head_dim, kTile) ||
+            !make_cache_map(&tmv, v_base, rows, d.head_dim, kTile)) {
             cached_k = cached_v = nullptr;
             *unsupported = true;
             return cudaSuccess;
         }
-        cached_k = k_cache;
-        cached_v = v_cache;
+        cached_k = k_base;
+        cached_v = v_base;
         cached_rows = rows;
         cached_d = d.head_dim;
     }
@@ -735,8 +774,8 @@ cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, i
     prm.k_new = static_cast<const __nv_bfloat16 *>(k_new);
     prm.v_new = static_cast<const __nv_bfloat16 *>(v_new);
     prm.new_pos = new_pos;
-    prm.k_cache = static_cast<__nv_bfloat16 *>(k_cache);
-    prm.v_cache = static_cast<__nv_bfloat16 *>(v_cache);
+    prm.k_cache = static_cast<__nv_bfloat16 *>(k_base);
+    prm.v_cache = static_cast<__nv_bfloat16 *>(v_base);
     prm.score = score;
     prm.pos = pos;
     prm.len = len;
@@ -745,10 +784,36 @@ cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, i
     prm.B = d.batch; prm.L = d.layers; prm.Hq = d.q_heads; prm.Hkv = d.kv_heads; prm.G = G;
     prm.C = d.capacity; prm.layer_begin = layer_begin; prm.chunk_cap = chunk_cap; prm.n_hint = nmax;
     prm.gamma = gamma;
+    prm.pv = pv;
     const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)d.head_dim);
     prm.scale_log2 = scale * 1.4426950408889634f;  // log2(e): exp(x) = 2^(x log2 e)
     return dispatch(d.head_dim, NT, pl.NS,
-                    [&](auto k) { return launch_t<decltype(k)>(tmk, tmv, prm, S, units, stream); });
+                    [&](auto k) { return launch_t<decltype(k)>(tmk, tmv, prm, S, units, stream, paged); });
+}
+
+}  // namespace
+
+cudaError_t launch_decode_mma(const voxzip_cache_desc &d, int32_t layer_begin, int32_t layer_count, const void *q,
+                              const void *k_new, const void *v_new, const int32_t *new_pos, void *k_cache,
+                              void *v_cache, float *score, int32_t *pos, int32_t *len, float gamma, float sm_scale,
+                              int32_t max_len, void *out, int32_t *status, cudaStream_t stream, bool *unsupported) {
+    const int64_t rows = (int64_t)d.batch * d.layers * d.kv_heads * d.capacity;
+    return launch_impl(d, k_cache, v_cache, rows, PageView{nullptr, nullptr, nullptr, 0}, layer_begin, layer_count, q,
+                       k_new, v_new, new_pos, score, pos, len, gamma, sm_scale, max_len, out, status, stream,
+                       unsupported);
+}
+
+bool decode_mma_paged_supported(const voxzip_cache_desc &d) { return decode_mma_supported(d); }
+
+cudaError_t launch_decode_mma_paged(const voxzip_cache_desc &d, const voxzip_paged_cache &pc, int32_t layer_begin,
+                                    int32_t layer_count, const void *q, const void *k_new, const void *v_new,
+                                    const int32_t *new_pos, float *score, int32_t *pos, int32_t *len, float gamma,
+                                    float sm_scale, int32_t max_len, void *out, int32_t *status, cudaStream_t stream,
+                                    bool *unsupported) {
+    const int64_t rows = (int64_t)pc.pages * kPageTokens;
+    return launch_impl(d, pc.k_pool, pc.v_pool, rows, PageView{pc.page_table, pc.free_pages, pc.free_count, pc.max_pages},
+                       layer_begin, layer_count, q, k_new, v_new, new_pos, score, pos, len, gamma, sm_scale, max_len,
+                       out, status, stream, unsupported);
 }
 
 }  // namespace voxzip

@@ -27,6 +27,7 @@
 // it, so no copy can read a row another one wrote.
 #include "common.cuh"
 #include "evict_policy.cuh"
+#include "paged.cuh"
 
 namespace voxzip {
 namespace {
@@ -45,6 +46,7 @@ struct EvictParams {
     int32_t B, L, Hkv, C, layer_begin, sink;
     int32_t budget_stride_b, budget_stride_l, history;
     float recent_frac;
+    PageView pv;  // paged instantiations only: K/V rows through the page table, pools as k/v_cache
 };
 
 // The unit's budget and its split into T sinks, M recent rows and N history rows.
@@ -152,7 +154,7 @@ __device__ void radix_pass(int shift, int lo, int hi, KeyFn key_of, RadixState &
     st = *shared_st;
 }
 
-template <typename T, int D>
+template <typename T, int D, bool kPaged>
 __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p) {
     constexpr int kVecPerRow = D * (int)sizeof(T) / 16;  // 16-byte vectors in one K (or V) row
     constexpr int kRows = kThreads * kStageVecs / (2 * kVecPerRow);
@@ -180,8 +182,10 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
     }
     float *sc = p.score + ui.cache_unit * p.C;
     int32_t *ps = p.pos + ui.cache_unit * p.C;
-    uint4 *kc = reinterpret_cast<uint4 *>(static_cast<T *>(p.k_cache) + ui.cache_unit * p.C * D);
-    uint4 *vc = reinterpret_cast<uint4 *>(static_cast<T *>(p.v_cache) + ui.cache_unit * p.C * D);
+    // K/V rows: the unit's slots (dense), or pool rows through the page table (paged).
+    uint4 *kc = reinterpret_cast<uint4 *>(static_cast<T *>(p.k_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
+    uint4 *vc = reinterpret_cast<uint4 *>(static_cast<T *>(p.v_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
+    auto slot_row = [&](int32_t slot) -> int64_t { return kPaged ? paged_row(p.pv, ui.cache_unit, slot) : slot; };
     const int32_t c_end = n - M;  // history candidates are slots [T, c_end)
 
     // Eq. 9: the N-th best history score, then (only if needed) the position cut among its ties.
@@ -242,7 +246,7 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
                 if (row < seg) {
                     const int src = src_list[row];
                     if (src != rank0 + row) {
-                        const uint4 *from = (w < kVecPerRow ? kc : vc) + (int64_t)src * kVecPerRow + (w % kVecPerRow);
+                        const uint4 *from = (w < kVecPerRow ? kc : vc) + slot_row(src) * kVecPerRow + (w % kVecPerRow);
                         asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
                                          (uint32_t)__cvta_generic_to_shared(&stage[st][v])),
                                      "l"(from)
@@ -275,7 +279,7 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
                     const int dst = rank0 + row;
                     if (src_list[row] != dst) {
                         uint4 *to = w < kVecPerRow ? kc : vc;
-                        to[(int64_t)dst * kVecPerRow + (w % kVecPerRow)] = stage[st][v];
+                        to[slot_row(dst) * kVecPerRow + (w % kVecPerRow)] = stage[st][v];
                     }
                 }
             }
@@ -302,9 +306,13 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
         rank0 += seg;
     }
     if (tid == 0) p.len[ui.cache_unit] = rank0;  // == budget
+    if constexpr (kPaged) {  // pages past the one holding slot bud go back to the pool
+        __syncthreads();
+        if (tid < 32) return_pages_warp(p.pv, ui.cache_unit, bud / kPageTokens + 1, n / kPageTokens + 1);
+    }
 }
 
-template <typename T, int D>
+template <typename T, int D, bool kPaged>
 __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictParams p) {
     constexpr int kVecPerRow = D * (int)sizeof(T) / 16;
     __shared__ int32_t holes[kSegment];
@@ -329,8 +337,9 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
     }
     float *sc = p.score + ui.cache_unit * p.C;
     int32_t *ps = p.pos + ui.cache_unit * p.C;
-    uint4 *kc = reinterpret_cast<uint4 *>(static_cast<T *>(p.k_cache) + ui.cache_unit * p.C * D);
-    uint4 *vc = reinterpret_cast<uint4 *>(static_cast<T *>(p.v_cache) + ui.cache_unit * p.C * D);
+    uint4 *kc = reinterpret_cast<uint4 *>(static_cast<T *>(p.k_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
+    uint4 *vc = reinterpret_cast<uint4 *>(static_cast<T *>(p.v_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
+    auto slot_row = [&](int32_t slot) -> int64_t { return kPaged ? paged_row(p.pv, ui.cache_unit, slot) : slot; };
 
     // Sinks: the T lowest positions (<= p_lo); recent window: the M highest (>= p_hi). Positions
     // of a unit are unique, so each select cuts exactly.
@@ -420,10 +429,10 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
         const int pairs = min(nh, nm);  // equal when positions are unique (then exactly `bud` rows are kept)
         if (pairs < nh && tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_POSITIONS);
         for (int v = tid; v < pairs * 2 * kVecPerRow; v += kThreads) {
-            const int row = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
+            const int r = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
             uint4 *base = w < kVecPerRow ? kc : vc;
             const int e = w % kVecPerRow;
-            base[(int64_t)holes[row] * kVecPerRow + e] = base[(int64_t)movers[row] * kVecPerRow + e];
+            base[slot_row(holes[r]) * kVecPerRow + e] = base[slot_row(movers[r]) * kVecPerRow + e];
         }
         for (int r = tid; r < pairs; r += kThreads) {
             sc[holes[r]] = sc[movers[r]];
@@ -438,14 +447,18 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
     for (int j = mcur + tid; j < n; j += kThreads) extra |= kept(j) ? 1 : 0;
     if (__syncthreads_or(extra) && tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_POSITIONS);
     if (tid == 0) p.len[ui.cache_unit] = bud;
+    if constexpr (kPaged) {  // pages past the one holding slot bud go back to the pool
+        __syncthreads();
+        if (tid < 32) return_pages_warp(p.pv, ui.cache_unit, bud / kPageTokens + 1, n / kPageTokens + 1);
+    }
 }
 
-template <typename T, int D>
+template <typename T, int D, bool kPaged = false>
 cudaError_t launch_t(const EvictParams &prm, int units, bool fill, cudaStream_t stream) {
     if (fill)
-        evict_fill_kernel<T, D><<<units, kThreads, 0, stream>>>(prm);
+        evict_fill_kernel<T, D, kPaged><<<units, kThreads, 0, stream>>>(prm);
     else
-        evict_kernel<T, D><<<units, kThreads, 0, stream>>>(prm);
+        evict_kernel<T, D, kPaged><<<units, kThreads, 0, stream>>>(prm);
     return cudaGetLastError();
 }
 
@@ -477,12 +490,33 @@ cudaError_t launch_evict_policy(const voxzip_cache_desc &d, int32_t layer_begin,
     prm.layer_begin = layer_begin; prm.sink = pol.sink; prm.recent_frac = pol.recent_frac;
     prm.budget_stride_b = pol.budget_stride_b; prm.budget_stride_l = pol.budget_stride_l;
     prm.history = pol.history;
+    prm.pv = PageView{nullptr, nullptr, nullptr, 0};
     const int units = layer_count * d.batch * d.kv_heads;
     const bool bf16 = d.dtype == VOXZIP_BF16, fill = pol.compaction == VOXZIP_COMPACT_FILL;
     if (d.head_dim == 128)
         return bf16 ? launch_t<__nv_bfloat16, 128>(prm, units, fill, stream)
                     : launch_t<float, 128>(prm, units, fill, stream);
     return bf16 ? launch_t<__nv_bfloat16, 64>(prm, units, fill, stream) : launch_t<float, 64>(prm, units, fill, stream);
+}
+
+cudaError_t launch_evict_paged(const voxzip_cache_desc &d, const voxzip_paged_cache &pc, int32_t layer_begin,
+                               int32_t layer_count, float *score, int32_t *pos, int32_t *len, const int32_t *budget,
+                               const voxzip_evict_policy &pol, int32_t *status, cudaStream_t stream) {
+    EvictParams prm;
+    prm.k_cache = pc.k_pool; prm.v_cache = pc.v_pool; prm.score = score; prm.pos = pos; prm.len = len;
+    prm.budget = budget; prm.status = status;
+    prm.B = d.batch; prm.L = d.layers; prm.Hkv = d.kv_heads; prm.C = d.capacity;
+    prm.layer_begin = layer_begin; prm.sink = pol.sink; prm.recent_frac = pol.recent_frac;
+    prm.budget_stride_b = pol.budget_stride_b; prm.budget_stride_l = pol.budget_stride_l;
+    prm.history = pol.history;
+    prm.pv = PageView{pc.page_table, pc.free_pages, pc.free_count, pc.max_pages};
+    const int units = layer_count * d.batch * d.kv_heads;
+    const bool bf16 = d.dtype == VOXZIP_BF16, fill = pol.compaction == VOXZIP_COMPACT_FILL;
+    if (d.head_dim == 128)
+        return bf16 ? launch_t<__nv_bfloat16, 128, true>(prm, units, fill, stream)
+                    : launch_t<float, 128, true>(prm, units, fill, stream);
+    return bf16 ? launch_t<__nv_bfloat16, 64, true>(prm, units, fill, stream)
+                : launch_t<float, 64, true>(prm, units, fill, stream);
 }
 
 }  // namespace voxzip

@@ -1,9 +1,11 @@
 """Host-side driver of the three C-ABI calls for one batch of sequences.
 
-A ``Session`` owns the device cache (K, V, score, pos, len), runs stage 1 once per request, then
-one decode step per generated token over all layers and an eviction every ``interval`` steps.
-It keeps a host-side upper bound on the cache length (read back once after stage 1) so that
-every decode launch is sized without a device-to-host sync.
+A ``Session`` owns the device cache (K, V, score, pos, len; or, paged, the page pools, the page
+table and the free-page stack), runs stage 1 once per request, then one decode step per
+generated token over all layers and an eviction every ``interval`` steps. It keeps a host-side
+upper bound on the cache length (read back once after stage 1) so that every decode launch is
+sized without a device-to-host sync; the decode loop of a request can therefore be captured once
+in a CUDA graph and replayed (``capture_loop``).
 """
 from __future__ import annotations
 
@@ -17,7 +19,8 @@ class Session:
     `compaction` select the eviction policy (see voxzip_evict_ex)."""
 
     def __init__(self, desc: N.CacheDesc, budget, gamma: float, *, sink: int = 4, recent_frac: float = 0.2,
-                 history: bool = True, compaction: str = "ordered", device="cuda", cache=None):
+                 history: bool = True, compaction: str = "ordered", device="cuda", cache=None,
+                 pages: int | None = None):
         self.desc = desc
         self.device = torch.device(device)
         self.gamma = float(gamma)
@@ -27,7 +30,13 @@ class Session:
         self.compaction = compaction
         self.budget = torch.tensor(budget, dtype=torch.int32, device=self.device)
         self.budget_host = [int(b) for b in self.budget.flatten().tolist()]
-        self.cache = cache if cache is not None else N.allocate_cache(desc, self.device)
+        self.paged = pages is not None
+        if cache is not None:
+            self.cache = cache
+        elif self.paged:
+            self.cache = N.allocate_paged_cache(desc, pages, self.device)
+        else:
+            self.cache = N.allocate_cache(desc, self.device)
         self.n_max = 0
         self.workspace = None
 
@@ -39,10 +48,15 @@ class Session:
         need = N.voxzip_anchor_fuse_workspace_size(self.desc, k_prefill.shape[3], span_start.numel())
         if self.workspace is None or self.workspace.numel() < need:
             self.workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=self.device)
-        N.voxzip_anchor_fuse(self.desc, k_prefill, v_prefill, in_len, audio_begin, audio_len, span_off,
-                             span_start, span_end, span_groups, c["k"], c["v"], c["score"], c["pos"], c["len"],
-                             slot_map=slot_map, anchor_k=anchor_k, anchor_v=anchor_v, workspace=self.workspace,
-                             stream=stream)
+        if self.paged:
+            N.voxzip_anchor_fuse_paged(self.desc, c, k_prefill, v_prefill, in_len, audio_begin, audio_len, span_off,
+                                       span_start, span_end, span_groups, slot_map=slot_map, anchor_k=anchor_k,
+                                       anchor_v=anchor_v, workspace=self.workspace, stream=stream)
+        else:
+            N.voxzip_anchor_fuse(self.desc, k_prefill, v_prefill, in_len, audio_begin, audio_len, span_off,
+                                 span_start, span_end, span_groups, c["k"], c["v"], c["score"], c["pos"], c["len"],
+                                 slot_map=slot_map, anchor_k=anchor_k, anchor_v=anchor_v, workspace=self.workspace,
+                                 stream=stream)
         if read_back:
             self.n_max = int(c["len"].max().item())
         else:
@@ -53,15 +67,23 @@ class Session:
         """One decode step for a layer range (all layers by default)."""
         c = self.cache
         lc = self.desc.layers if layer_count is None else layer_count
-        N.voxzip_decode_step(self.desc, layer_begin, lc, q, k_new, v_new, new_pos, c["k"], c["v"], c["score"],
-                             c["pos"], c["len"], self.gamma, out, max_len=self.n_max + 1, stream=stream)
+        if self.paged:
+            N.voxzip_decode_step_paged(self.desc, c, layer_begin, lc, q, k_new, v_new, new_pos, self.gamma, out,
+                                       max_len=self.n_max + 1, stream=stream)
+        else:
+            N.voxzip_decode_step(self.desc, layer_begin, lc, q, k_new, v_new, new_pos, c["k"], c["v"], c["score"],
+                                 c["pos"], c["len"], self.gamma, out, max_len=self.n_max + 1, stream=stream)
         if layer_begin + lc == self.desc.layers:
             self.n_max += 1
 
     def evict(self, *, layer_begin=0, layer_count=None, stream=None):
         c = self.cache
         lc = self.desc.layers if layer_count is None else layer_count
-        if self.history and self.compaction == "ordered" and self.budget.dim() == 1:
+        if self.paged:
+            N.voxzip_evict_paged(self.desc, c, layer_begin, lc, self.budget, sink=self.sink,
+                                 recent_frac=self.recent_frac, history=self.history, compaction=self.compaction,
+                                 stream=stream)
+        elif self.history and self.compaction == "ordered" and self.budget.dim() == 1:
             N.voxzip_evict(self.desc, layer_begin, lc, c["k"], c["v"], c["score"], c["pos"], c["len"], self.budget,
                            sink=self.sink, recent_frac=self.recent_frac, stream=stream)
         else:
@@ -70,3 +92,41 @@ class Session:
                               compaction=self.compaction, stream=stream)
         if layer_begin + lc == self.desc.layers:
             self.n_max = min(self.n_max, max(self.budget_host))
+
+    # decode loop in a CUDA graph ---------------------------------------------------------------------
+    def capture_loop(self, q, k_new, v_new, new_pos, out, interval: int, *, launch_events=None):
+        """Captures the decode loop of one request: step t (1-based) decodes with q[t-1], k_new[t-1],
+        v_new[t-1], new_pos[t-1] into out[t-1], and evicts when t % interval == 0. Call it right
+        after a prefill of the request's shape (it starts from that cache length bound); replaying
+        the returned graph after each later prefill of the same shape runs the whole loop with one
+        host call. With `launch_events` (a list), a pair of timing events (created with
+        external=True) around every decode and every eviction launch is captured too and appended
+        as ("decode" | "evict", start, end)."""
+        n0 = self.n_max
+        stream = torch.cuda.Stream(device=self.device)
+        stream.wait_stream(torch.cuda.current_stream(self.device))
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.stream(stream):
+            with torch.cuda.graph(graph, stream=stream):
+                for t in range(1, q.shape[0] + 1):
+                    ev = None
+                    if launch_events is not None:
+                        ev = (torch.cuda.Event(enable_timing=True, external=True),
+                              torch.cuda.Event(enable_timing=True, external=True))
+                        ev[0].record()
+                    self.decode(q[t - 1], k_new[t - 1], v_new[t - 1], new_pos[t - 1], out[t - 1])
+                    if ev is not None:
+                        ev[1].record()
+                        launch_events.append(("decode",) + ev)
+                    if t % interval == 0:
+                        if launch_events is not None:
+                            ev = (torch.cuda.Event(enable_timing=True, external=True),
+                                  torch.cuda.Event(enable_timing=True, external=True))
+                            ev[0].record()
+                        self.evict()
+                        if launch_events is not None:
+                            ev[1].record()
+                            launch_events.append(("evict",) + ev)
+        torch.cuda.current_stream(self.device).wait_stream(stream)
+        self.n_max = n0
+        return graph

@@ -70,16 +70,32 @@ def unit_budget(w, policy, b, l):
     return int(bl[b][l]) if bl is not None else int(w.budget[b])
 
 
+def unit_rows(c, sel, which, D):
+    """K or V rows [k][C][D] of the selected units (bi, li, hi): the dense cache, or gathered from a
+    paged cache's pool through its page table (slots without a page read pool row 0)."""
+    bi, li, hi = sel
+    if which in c:
+        return c[which][bi, li, hi]
+    tab = c["page_table"][bi, li, hi]                       # [k][max_pages]
+    C = tab.shape[1] * 64
+    slots = torch.arange(C, device=tab.device)
+    rows = tab[:, slots // 64].clamp(min=0).long() * 64 + slots % 64
+    return c[which + "_pool"].view(-1, D)[rows]
+
+
 def gpu_run(w, inp, sample, steps=None, anchors=None, policy=None):
     """The whole path on the GPU through the C ABI; records the sampled units. `policy` (optional)
-    holds history (bool), compaction ("ordered" / "fill") and budget_bl ([B][L] budgets)."""
+    holds history (bool), compaction ("ordered" / "fill"), budget_bl ([B][L] budgets) and pages
+    (a paged cache of that many pages)."""
     S = w.steps if steps is None else steps
     dev = inp["k_pre"].device
     B, L, Hq, H, D, G = w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.group
-    desc = CacheDesc(B, L, Hq, H, D, w.capacity, w.dtype)
     pol = policy or {}
+    cap = w.capacity if pol.get("pages") is None else (w.capacity + 63) // 64 * 64   # paged: whole pages
+    desc = CacheDesc(B, L, Hq, H, D, cap, w.dtype)
     sess = Session(desc, pol.get("budget_bl", w.budget), w.gamma, sink=w.sink, recent_frac=w.recent_frac,
-                   history=pol.get("history", True), compaction=pol.get("compaction", "ordered"), device=dev)
+                   history=pol.get("history", True), compaction=pol.get("compaction", "ordered"), device=dev,
+                   pages=pol.get("pages"))
     sp = inp["spans"]
     i32 = lambda a: torch.as_tensor(np.asarray(a), dtype=torch.int32, device=dev)
     slot_map = torch.full((B, w.stride), -1, dtype=torch.int32, device=dev)
@@ -93,8 +109,9 @@ def gpu_run(w, inp, sample, steps=None, anchors=None, policy=None):
     li = torch.tensor([u[1] for u in sample], device=dev)
     hi = torch.tensor([u[2] for u in sample], device=dev)
     ar = torch.arange(len(sample), device=dev)
-    rec = dict(stage1_len=c["len"][bi, li, hi].cpu().numpy(), stage1_k=c["k"][bi, li, hi].cpu(),
-               stage1_v=c["v"][bi, li, hi].cpu(), stage1_pos=c["pos"][bi, li, hi].cpu().numpy(),
+    sel = (bi, li, hi)
+    rec = dict(stage1_len=c["len"][bi, li, hi].cpu().numpy(), stage1_k=unit_rows(c, sel, "k", D).cpu(),
+               stage1_v=unit_rows(c, sel, "v", D).cpu(), stage1_pos=c["pos"][bi, li, hi].cpu().numpy(),
                slot_map=slot_map.cpu().numpy())
     out = torch.empty(L, B, Hq, D, dtype=w.dtype, device=dev)
     outs, sb, lb, kp = [], [], [], []
@@ -115,8 +132,9 @@ def gpu_run(w, inp, sample, steps=None, anchors=None, policy=None):
     rec["len"] = c["len"][bi, li, hi].cpu().numpy()
     rec["score"] = c["score"][bi, li, hi].cpu().numpy()
     rec["pos"] = c["pos"][bi, li, hi].cpu().numpy()
-    rec["k"] = c["k"][bi, li, hi].cpu()
-    rec["v"] = c["v"][bi, li, hi].cpu()
+    rec["k"] = unit_rows(c, sel, "k", D).cpu()
+    rec["v"] = unit_rows(c, sel, "v", D).cpu()
+    rec["session"] = sess
     return rec
 
 
