@@ -54,6 +54,9 @@ def parse_args():
     p.add_argument("--cpu-units", type=int, default=0, help="units in the oracle sample (0: one per core)")
     p.add_argument("--compaction", choices=["ordered", "fill"], default="ordered",
                    help="eviction compaction: ordered (Eq. 7-8, default) or hole filling")
+    p.add_argument("--paged", action="store_true", help="K/V in a paged cache (pages of 64 rows)")
+    p.add_argument("--graph", action="store_true",
+                   help="replay the decode loop of a request from one CUDA graph (stage 1 stays eager)")
     p.add_argument("--part", choices=["path", "embed"], default="path",
                    help="path: the KV-compression path (default); embed: embedding-level stage 1")
     return p.parse_args()
@@ -212,7 +215,7 @@ def evict_bytes(w, n_before, moved_rows):
 # ----------------------------------------------------------------------------- GPU arm
 
 class Runner:
-    def __init__(self, w, device, compaction="ordered"):
+    def __init__(self, w, device, compaction="ordered", paged=False):
         from paper_2608_08569_gb300 import CacheDesc
         from paper_2608_08569_gb300 import workloads as W
         from paper_2608_08569_gb300.session import Session
@@ -224,17 +227,40 @@ class Runner:
                           i32(self.spans.start), i32(self.spans.end), i32(self.spans.groups))
         self.k_pre, self.v_pre = W.make_prefill(w, device)
         self.q, self.kn, self.vn, self.npos = W.make_steps(w, device)
-        self.desc = CacheDesc(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.capacity, w.dtype)
+        cap = (w.capacity + 63) // 64 * 64 if paged else w.capacity
+        self.desc = CacheDesc(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, cap, w.dtype)
+        # a paged pool as large as the dense cache: the footprint reported is the pages in use
+        self.pages = w.units * (cap // 64) if paged else None
         self.sess = Session(self.desc, w.budget, w.gamma, sink=w.sink, recent_frac=w.recent_frac,
-                            compaction=compaction, device=device)
+                            compaction=compaction, device=device, pages=self.pages)
+        self.graph = None
         self.out = torch.empty(w.steps, w.layers, w.batch, w.q_heads, w.head_dim, dtype=w.dtype, device=device)
 
-    def request(self, timers=None, lengths=None, evict_timers=None, moved=None):
-        """One request: stage 1, then every decode step with evictions. With `timers` (and
-        `evict_timers`), records a CUDA event pair around every decode (evict) launch on the launch
-        stream. With `moved`, records per eviction the units' lengths and moved rows (this syncs)."""
+    def capture(self):
+        """Captures the decode loop (with timing events around every launch) after a stage 1."""
         w, s = self.w, self.sess
         s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
+        self.graph_events = []
+        self.graph = s.capture_loop(self.q, self.kn, self.vn, self.npos, self.out, w.interval,
+                                    launch_events=self.graph_events)
+
+    def request_graph(self):
+        """One request with the decode loop replayed from the graph."""
+        s = self.sess
+        s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
+        self.graph.replay()
+
+    def request(self, timers=None, lengths=None, evict_timers=None, moved=None, pages=None):
+        """One request: stage 1, then every decode step with evictions. With `timers` (and
+        `evict_timers`), records a CUDA event pair around every decode (evict) launch on the launch
+        stream. With `moved`, records per eviction the units' lengths and moved rows (this syncs).
+        With `pages` (paged cache), records the pages in use after stage 1 and around the first
+        eviction (this syncs)."""
+        w, s = self.w, self.sess
+        s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
+        if pages is not None:
+            from paper_2608_08569_gb300 import paged_pages_in_use
+            pages.append(paged_pages_in_use(s.cache))
         n = s.cache["len"][:, 0, 0].tolist() if lengths is not None else None
         stream = torch.cuda.current_stream()
         for t in range(1, w.steps + 1):
@@ -260,7 +286,11 @@ class Runner:
                     f0 = torch.cuda.Event(enable_timing=True)
                     f1 = torch.cuda.Event(enable_timing=True)
                     f0.record(stream)
+                if pages is not None and t == w.interval:
+                    pages.append(paged_pages_in_use(s.cache))
                 s.evict()
+                if pages is not None and t == w.interval:
+                    pages.append(paged_pages_in_use(s.cache))
                 if evict_timers is not None:
                     f1.record(stream)
                     evict_timers.append((f0, f1))
@@ -288,12 +318,17 @@ def gpu_arm(args, rank, world, local):
     w = W.CONFIGS[args.workload]
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
-    r = Runner(w, dev, compaction=args.compaction)
+    r = Runner(w, dev, compaction=args.compaction, paged=args.paged)
     for _ in range(args.warmup):
         r.request()
+    lengths = []
+    if args.graph:
+        r.capture()
+        r.request(lengths=lengths)   # the lengths of one request (same in every replay)
+        r.request_graph()
     torch.cuda.synchronize()
     barrier(world)
-    timers, lengths, ev_timers = [], [], []
+    timers, ev_timers = [], []
     with ClockSampler(local) as clk:
         torch.cuda.synchronize()
         barrier(world)
@@ -301,10 +336,16 @@ def gpu_arm(args, rank, world, local):
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record()
         for k in range(args.steps):
-            r.request(timers=timers, lengths=lengths if k == 0 else None, evict_timers=ev_timers)
+            if args.graph:
+                r.request_graph()
+            else:
+                r.request(timers=timers, lengths=lengths if k == 0 else None, evict_timers=ev_timers)
         e1.record()
         torch.cuda.synchronize()
         barrier(world)
+    if args.graph:  # per-launch times of the last replay, as if every replay took them
+        timers = [(a, b) for kind, a, b in r.graph_events if kind == "decode"] * args.steps
+        ev_timers = [(a, b) for kind, a, b in r.graph_events if kind == "evict"] * args.steps
     ms = e0.elapsed_time(e1)
     ms_max = max_over_ranks(ms, world)
     total_steps = world * args.steps * w.steps
@@ -339,12 +380,12 @@ def gpu_arm(args, rank, world, local):
         t = sum(timers[i][0].elapsed_time(timers[i][1]) for i in ids)
         if t > 0:
             roofline[f"achieved_{name}"] = round(b / (t / 1000.0) / 1e9, 1)
-    # kernels per request: 3 stage-1 kernels, one decode launch per step, one evict per interval
-    gpu_launches = args.steps * (3 + w.steps + n_evict)
+    # kernels per request: 3 stage-1 kernels (5 paged), one decode launch per step, one evict per interval
+    gpu_launches = args.steps * ((5 if args.paged else 3) + w.steps + n_evict)
 
     # The eviction kernel against the same peak: bytes from an untimed replay of one request.
-    moved = []
-    r.request(moved=moved)
+    moved, pages = [], ([] if args.paged else None)
+    r.request(moved=moved, pages=pages)
     torch.cuda.synchronize()
     ev_bytes = sum(evict_bytes(w, nb, mv) for nb, mv in moved)
     ev_ms = sum(a.elapsed_time(b) for a, b in ev_timers)
@@ -378,7 +419,14 @@ def gpu_arm(args, rank, world, local):
                    "q_heads": w.q_heads, "kv_heads": w.kv_heads, "head_dim": w.head_dim,
                    "prompt_tokens": list(sorted(set(w.in_len))), "budget": list(sorted(set(w.budget))),
                    "gamma": w.gamma, "decode_steps_per_request": w.steps, "evict_interval": w.interval,
-                   "compaction": args.compaction,
+                   "compaction": args.compaction, "graph": bool(args.graph),
+                   "paged": None if not args.paged else {
+                       "page_rows": 64, "pool_pages": r.pages,
+                       "bytes_per_page": 2 * 64 * w.head_dim * (2 if w.dtype == torch.bfloat16 else 4),
+                       "pages_after_stage1": pages[0], "pages_before_first_evict": pages[1],
+                       "pages_after_first_evict": pages[2],
+                       "dense_cache_bytes": w.units * r.desc.capacity * 2 * w.head_dim *
+                                            (2 if w.dtype == torch.bfloat16 else 4)},
                    "parallelism": f"replicas x{world} (independent units, no collective)",
                    "l2": "inputs larger than L2 (decode reads ~0.9-7 GB per launch, L2 is 129 MB)"},
         "roofline": roofline, "roofline_evict": roofline_evict, "gpu_launches": gpu_launches, "clocks": clocks,
@@ -417,7 +465,10 @@ def e2e_leg(r, args):
         r.q.copy_(h["q"], non_blocking=True)
         r.kn.copy_(h["kn"], non_blocking=True)
         r.vn.copy_(h["vn"], non_blocking=True)
-        r.request()
+        if r.graph is not None:
+            r.request_graph()
+        else:
+            r.request()
         h_out.copy_(r.out, non_blocking=True)
 
     request()
