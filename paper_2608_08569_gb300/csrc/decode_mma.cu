@@ -142,6 +142,24 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         const int rows = min(kStages * kTile, p.C - est_j0);
         if (rows > 0) ptx::prefetch_l2(p.k_cache + (row_base + est_j0) * D, (uint32_t)rows * D * 2);
     }
+    // Paged: before the length is known, the producer reads the page-table entries of the range the
+    // launch's length hint predicts and pulls those tiles into L2 (kept when the prediction holds).
+    int est_j0 = -1, est_tiles = 0;
+    if constexpr (kPaged) {
+        if (warp == kConsumerWarps) {
+            const int est_chunk = ((p.n_hint + S - 1) / S + kTile - 1) / kTile * kTile;
+            est_j0 = rank * est_chunk;
+            est_tiles = max(0, min(est_chunk, p.n_hint - est_j0) + kTile - 1) / kTile;
+            est_tiles = min(est_tiles, p.pv.max_pages - est_j0 / kTile);
+            const int32_t *trow = p.pv.table + ui.cache_unit * p.pv.max_pages + est_j0 / kTile;
+            for (int t = lane; t < est_tiles; t += 32) {
+                const int32_t page = trow[t];
+                tile_rows[t] = page * kTile;
+                if (t < kStages && page >= 0)
+                    ptx::prefetch_l2(p.k_cache + (int64_t)page * kTile * D, (uint32_t)kTile * D * 2);
+            }
+        }
+    }
     // The queries do not depend on the length: load them first. Q^T is the B operand:
     // b0b1 = Q[head][16ks + 2qd .. +1], b2b3 = Q[head][16ks + 8 + 2qd .. +1].
     uint32_t qb[NT][kKSteps][2];
@@ -225,8 +243,10 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     if (warp == kConsumerWarps) {
         // ------------------------------------------------------------- producer
         if constexpr (kPaged) {  // the pool row of every tile of the range (j0 is page-aligned)
-            const int32_t *trow = p.pv.table + ui.cache_unit * p.pv.max_pages + j0 / kTile;
-            for (int t = lane; t < ntiles; t += 32) tile_rows[t] = trow[t] * kTile;
+            if (j0 != est_j0 || ntiles > est_tiles) {
+                const int32_t *trow = p.pv.table + ui.cache_unit * p.pv.max_pages + j0 / kTile;
+                for (int t = lane; t < ntiles; t += 32) tile_rows[t] = trow[t] * kTile;
+            }
             __syncwarp();
         }
         if (lane == 0 && ntiles > 0) {

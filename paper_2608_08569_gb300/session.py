@@ -101,7 +101,8 @@ class Session:
         the returned graph after each later prefill of the same shape runs the whole loop with one
         host call. With `launch_events` (a list), a pair of timing events (created with
         external=True) around every decode and every eviction launch is captured too and appended
-        as ("decode" | "evict", start, end)."""
+        as ("decode" | "evict", start, end); the graph records into them on every replay, so they
+        must outlive it."""
         n0 = self.n_max
         stream = torch.cuda.Stream(device=self.device)
         stream.wait_stream(torch.cuda.current_stream(self.device))
