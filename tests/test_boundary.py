@@ -118,3 +118,56 @@ def test_binding_rejects_host_tensors():
     with pytest.raises(ValueError):
         V.voxzip_evict(desc, 0, 1, t, t, torch.zeros(1, 1, 1, 8), torch.zeros(1, 1, 1, 8, dtype=torch.int32),
                        torch.zeros(1, 1, 1, dtype=torch.int32), torch.zeros(1, dtype=torch.int32))
+
+
+# --------------------------------------------------------------------- the NEXT rows' entry points
+
+def _paged(**kw):
+    import paper_2608_08569_gb300 as V
+    base = dict(k_pool=256, v_pool=256, page_table=256, free_pages=256, free_count=256, pages=64, max_pages=1)
+    base.update(kw)
+    return V._native._Paged(*[base[k] for k in ("k_pool", "v_pool", "page_table", "free_pages", "free_count",
+                                                   "pages", "max_pages")])
+
+
+def _policy(**kw):
+    import paper_2608_08569_gb300 as V
+    base = dict(sink=4, recent_frac=0.2, history=1, budget_stride_b=1, budget_stride_l=0, compaction=0)
+    base.update(kw)
+    return V._native._EvictPolicy(*[base[k] for k in ("sink", "recent_frac", "history", "budget_stride_b",
+                                                         "budget_stride_l", "compaction")])
+
+
+@pytest.mark.parametrize("kw", [dict(compaction=2), dict(history=3), dict(budget_stride_b=-1), dict(sink=-1),
+                                dict(recent_frac=1.5)])
+def test_evict_policy_is_validated(L, kw):
+    d, pol = _desc(), _policy(**kw)
+    assert L.voxzip_evict_ex(ctypes.byref(d), 0, 1, P, P, P, P, P, P, ctypes.byref(pol), None) == 1
+    assert L.voxzip_evict_ex(ctypes.byref(d), 0, 1, P, P, P, P, P, P, None, None) == 1
+
+
+@pytest.mark.parametrize("kw", [dict(max_pages=2), dict(pages=1), dict(k_pool=0), dict(k_pool=264)])
+def test_paged_cache_is_validated(L, kw):
+    """capacity (64 here) must be 64 x max_pages, the pool must hold a page per unit, pools are
+    non-null and 16-byte aligned."""
+    d, pc = _desc(), _paged(**kw)
+    assert L.voxzip_decode_step_paged(ctypes.byref(d), ctypes.byref(pc), 0, 1, P, P, P, P, P, P, P, 0.9, 0.0, 0,
+                                      P, None) == 1
+    assert L.voxzip_paged_init(ctypes.byref(d), ctypes.byref(pc), P, None) == 1
+    pol = _policy()
+    assert L.voxzip_evict_paged(ctypes.byref(d), ctypes.byref(pc), 0, 1, P, P, P, P, ctypes.byref(pol), None) == 1
+
+
+def test_paged_init_needs_lengths(L):
+    d, pc = _desc(), _paged()
+    assert L.voxzip_paged_init(ctypes.byref(d), ctypes.byref(pc), None, None) == 1
+
+
+@pytest.mark.parametrize("d_model,dtype,keep", [(12, 1, 1), (6, 0, 1), (64, 1, 2), (0, 1, 1)])
+def test_embed_fuse_is_validated(L, d_model, dtype, keep):
+    import paper_2608_08569_gb300 as V
+    e = V._native._EmbedDesc(2, d_model, 64, dtype)
+    assert L.voxzip_embed_fuse_workspace_size(ctypes.byref(e), 100, 3) == 0 or keep == 2
+    rc = L.voxzip_embed_fuse(ctypes.byref(e), P, 100, P, P, P, P, 0, None, None, None, None, 0, keep, P, P, P,
+                             None, P, 1 << 20, None)
+    assert rc == 1
