@@ -53,7 +53,7 @@ def _gather_text(segs, text_all, idx):
     return out
 
 
-def _run_gpu(w, e_in, spans, e_text, keep_bg, capacity=None):
+def _run_gpu(w, e_in, spans, e_text, keep_bg, capacity=None, with_slot_map=True):
     off, st, en, gr, _ = spans
     C = capacity or w.capacity
     dev = e_in.device
@@ -61,7 +61,7 @@ def _run_gpu(w, e_in, spans, e_text, keep_bg, capacity=None):
     out = torch.full((w.batch, C, w.d_model), float("nan"), dtype=w.dtype, device=dev)
     pos = torch.full((w.batch, C), -7, dtype=torch.int32, device=dev)
     ln = torch.full((w.batch,), -7, dtype=torch.int32, device=dev)
-    sm = torch.full((w.batch, w.stride), -7, dtype=torch.int32, device=dev)
+    sm = torch.full((w.batch, w.stride), -7, dtype=torch.int32, device=dev) if with_slot_map else None
     voxzip_embed_fuse(EmbedDesc(w.batch, w.d_model, C, w.dtype), e_in, i32(w.in_len), i32([w.audio_begin] * w.batch),
                       i32(w.audio_len), i32(off), i32(st), i32(en), i32(gr), out, pos, ln, e_text=e_text,
                       keep_background=keep_bg, slot_map=sm)
@@ -164,3 +164,22 @@ def test_embed_edge_cases():
     assert bits & DEV_BAD_SPANS and bits & DEV_CAPACITY
     assert int(ln[0]) == 0 and int(ln[2]) == 0 and int(ln[1]) == 56 - 10 + 2
     assert voxzip_get_status() == 0
+
+
+@pytest.mark.parametrize("name", ["embed_tiny", "embed_short"])
+@pytest.mark.parametrize("keep_bg", [True, False])
+def test_embed_fuse_without_slot_map_gives_the_same_rows(name, keep_bg):
+    """Without a slot map the per-token plan is skipped; the rows, positions and lengths are the
+    same bits."""
+    w = W.EMBED_CONFIGS[name]
+    segs = W.make_segments(w)
+    e_in = W.make_embeddings(w, "cuda")
+    spans = _spans(w, segs, voxzip_segments_to_spans)
+    e_text = _gather_text(segs, W.make_text_embeddings(w, segs, "cuda"), spans[4])
+    a = _run_gpu(w, e_in, spans, e_text, keep_bg, with_slot_map=True)
+    b = _run_gpu(w, e_in, spans, e_text, keep_bg, with_slot_map=False)
+    assert voxzip_get_status() == 0
+    assert torch.equal(a[2], b[2])
+    for bb in range(w.batch):
+        n = int(a[2][bb])
+        assert torch.equal(a[0][bb, :n], b[0][bb, :n]) and torch.equal(a[1][bb, :n], b[1][bb, :n])
