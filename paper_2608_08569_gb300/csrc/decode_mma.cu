@@ -7,10 +7,12 @@
 // into a shared-memory ring guarded by mbarriers; four consumer warps take 16 tokens of every tile:
 //   phase K  S = K_tile Q^T on the tensor cores (mma.sync m16n8k16, tokens as M, the group's
 //            query heads as N); scaled logits kept in shared memory; a running per-head maximum
-//            and normaliser (online softmax statistics).
-//   phase V p = 2^(logit - max_cta); O^T += V_tile^T P^T on the tensor cores. A CTA that holds the
+//            and normaliser (online softmax statistics; kept only when S = 1).
+//   phase V  p = 2^(logit - max_cta); O^T += V_tile^T P^T on the tensor cores. A CTA that holds the
 //            whole unit (S = 1) already has the final statistics: it rewrites the scores tile by
 //            tile as gamma * s + sum_h p_h / Z_h. In a cluster p is kept in shared memory instead.
+// As each tile issues, the tile one ring-depth ahead is requested into L2 (bulk prefetch), so an
+// SM keeps more bytes in flight than its rings hold.
 // In a cluster, one exchange through distributed shared memory then gives the unit's per-head
 // maximum and normaliser: every CTA rewrites its tokens' scores and combines one slice of the
 // G x D outputs from all CTAs' partials. (Exchanging the statistics between the two phases instead
@@ -32,6 +34,9 @@ namespace {
 
 #ifndef VOXZIP_DECODE_WARPS
 #define VOXZIP_DECODE_WARPS 4      // consumer warps per CTA (16 tokens of every tile each)
+#endif
+#ifndef VOXZIP_DECODE_L2_AHEAD
+#define VOXZIP_DECODE_L2_AHEAD 1           // tiles past the ring requested into L2 as each tile issues
 #endif
 #ifndef VOXZIP_DECODE_CTA_FIXED_US
 #define VOXZIP_DECODE_CTA_FIXED_US 5.0     // a CTA's fixed latency: first tiles, exit
@@ -266,6 +271,20 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
 #pragma unroll
                 for (int h = 0; h < kHalves; ++h)
                     ptx::tma_load_2d(dst + h * kBoxBytes, is_k ? &tmk : &tmv, h * kBoxCols, y, &full[s]);
+                // L2 look-ahead: the tile that will issue once the ring turns over starts toward L2
+                // now. It costs no shared memory and keeps more of the SM's bytes in flight; its TMA
+                // load then hits L2.
+                if (VOXZIP_DECODE_L2_AHEAD > 0) {
+                    const int ia = i + kStages + VOXZIP_DECODE_L2_AHEAD - 1;
+                    if (ia < 2 * ntiles) {
+                        const bool ak = ia < ntiles;
+                        const int at = ak ? ia : ia - ntiles;
+                        const int rows = min(kTile, cnt - at * kTile);
+                        const int64_t row0 = kPaged ? (int64_t)tile_rows[at] : row_base + j0 + (int64_t)at * kTile;
+                        if (rows > 0)
+                            ptx::prefetch_l2((ak ? p.k_cache : p.v_cache) + row0 * D, (uint32_t)rows * D * 2);
+                    }
+                }
             }
         }
         __syncwarp();  // reconverge the producer warp
