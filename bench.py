@@ -5,9 +5,12 @@ One bench step is one request of the workload run through the whole path via the
 stage-1 fusion of the resident prefilled K/V, then every decode step over all 48 layers
 (fused append + GQA attention + decayed-score update) with an eviction every `interval` steps.
 The reported value is decode steps per second of the whole job (each decode step advances every
-sequence of the batch by one token through all layers), stage 1 and evictions included.
+sequence of the batch by one token through all layers), stage 1 and evictions included. By
+default each request's decode loop (its decodes and evictions) replays from one CUDA graph
+captured once, each launch a programmatic dependent of the one before; stage 1 runs eagerly.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--workload stress] [--impl voxzip|reference]
+                  [--loop graph|eager] [--compaction ordered|fill] [--paged]
   python bench.py --part embed [--steps K] [--warmup W]
 
 `--part embed` measures stage 1 where the paper runs it instead: ASR segments of 4 x 60 min of
@@ -55,8 +58,10 @@ def parse_args():
     p.add_argument("--compaction", choices=["ordered", "fill"], default="ordered",
                    help="eviction compaction: ordered (Eq. 7-8, default) or hole filling")
     p.add_argument("--paged", action="store_true", help="K/V in a paged cache (pages of 64 rows)")
-    p.add_argument("--graph", action="store_true",
-                   help="replay the decode loop of a request from one CUDA graph (stage 1 stays eager)")
+    p.add_argument("--loop", choices=["graph", "eager"], default="graph",
+                   help="graph (default): each request's decode loop replays from one captured CUDA graph, "
+                        "stage 1 stays eager; eager: one host launch per decode and eviction")
+    p.add_argument("--graph", action="store_true", help="same as --loop graph")
     p.add_argument("--part", choices=["path", "embed"], default="path",
                    help="path: the KV-compression path (default); embed: embedding-level stage 1")
     return p.parse_args()
@@ -237,12 +242,16 @@ class Runner:
         self.out = torch.empty(w.steps, w.layers, w.batch, w.q_heads, w.head_dim, dtype=w.dtype, device=device)
 
     def capture(self):
-        """Captures the decode loop (with timing events around every launch) after a stage 1."""
+        """Captures the decode loop twice after a stage 1: `graph` as it runs (back-to-back launches,
+        each a programmatic dependent of the one before), and `graph_timed` with timing events
+        around every launch (events between launches also separate them), for the roofline."""
         w, s = self.w, self.sess
         s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
+        self.graph = s.capture_loop(self.q, self.kn, self.vn, self.npos, self.out, w.interval)
+        s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
         self.graph_events = []
-        self.graph = s.capture_loop(self.q, self.kn, self.vn, self.npos, self.out, w.interval,
-                                    launch_events=self.graph_events)
+        self.graph_timed = s.capture_loop(self.q, self.kn, self.vn, self.npos, self.out, w.interval,
+                                          launch_events=self.graph_events)
 
     def request_graph(self):
         """One request with the decode loop replayed from the graph."""
@@ -336,14 +345,17 @@ def gpu_arm(args, rank, world, local):
         e1 = torch.cuda.Event(enable_timing=True)
         e0.record()
         for k in range(args.steps):
-            if args.graph:
+            if args.graph and k < args.steps - 1:
                 r.request_graph()
+            elif args.graph:  # the last request replays the instrumented copy: per-launch events
+                r.sess.prefill(r.k_pre, r.v_pre, *r.span_args[:3], *r.span_args[3:])
+                r.graph_timed.replay()
             else:
                 r.request(timers=timers, lengths=lengths if k == 0 else None, evict_timers=ev_timers)
         e1.record()
         torch.cuda.synchronize()
         barrier(world)
-    if args.graph:  # per-launch times of the last replay, as if every replay took them
+    if args.graph:  # per-launch times of the instrumented replay, as if every replay took them
         timers = [(a, b) for kind, a, b in r.graph_events if kind == "decode"] * args.steps
         ev_timers = [(a, b) for kind, a, b in r.graph_events if kind == "evict"] * args.steps
     ms = e0.elapsed_time(e1)
@@ -420,6 +432,12 @@ def gpu_arm(args, rank, world, local):
                    "prompt_tokens": list(sorted(set(w.in_len))), "budget": list(sorted(set(w.budget))),
                    "gamma": w.gamma, "decode_steps_per_request": w.steps, "evict_interval": w.interval,
                    "compaction": args.compaction, "graph": bool(args.graph),
+                   "loop": "graph" if args.graph else "eager",
+                   "roofline_timing": ("CUDA events around every launch of the last timed request, which "
+                                       "replays an instrumented copy of the graph (events between launches "
+                                       "keep them from overlapping, so the others replay without)")
+                                      if args.graph else
+                                      "CUDA events around every launch inside the timed region",
                    "paged": None if not args.paged else {
                        "page_rows": 64, "pool_pages": r.pages,
                        "bytes_per_page": 2 * 64 * w.head_dim * (2 if w.dtype == torch.bfloat16 else 4),
@@ -472,12 +490,13 @@ def e2e_leg(r, args):
             getattr(r, n).copy_(host[n])
         for d, h in zip(r.span_args, host_spans):
             d.copy_(h)
+        timed0 = r.graph_timed
         r.capture()
         graphs[1] = r.graph
         # A graph records into its timing events on every replay: they, and the buffers the graph
         # reads, must live as long as the graph does.
-        r.keep_alive = (graphs, sets, r.graph_events)
-        r.graph_events = events0
+        r.keep_alive = (graphs, sets, r.graph_timed, r.graph_events)
+        r.graph_events, r.graph_timed = events0, timed0
         torch.cuda.synchronize()
     up, down = torch.cuda.Stream(), torch.cuda.Stream()
     comp = torch.cuda.current_stream()
@@ -822,6 +841,7 @@ def embed_cpu_sample(r, cols=16):
 
 def main():
     args = parse_args()
+    args.graph = args.graph or args.loop == "graph"
     rank, world, local = dist_setup()
     if args.part == "embed" and args.impl != "reference":
         res = embed_arm(args, rank, world, local)

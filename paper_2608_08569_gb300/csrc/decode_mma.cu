@@ -12,7 +12,9 @@
 //            whole unit (S = 1) already has the final statistics: it rewrites the scores tile by
 //            tile as gamma * s + sum_h p_h / Z_h. In a cluster p is kept in shared memory instead.
 // As each tile issues, the tile one ring-depth ahead is requested into L2 (bulk prefetch), so an
-// SM keeps more bytes in flight than its rings hold.
+// SM keeps more bytes in flight than its rings hold. Launches are programmatic dependents of the
+// previous kernel on the stream: a CTA sets up (barriers, the L2 prefetch of its first tiles)
+// while that kernel drains, then waits for it before its first dependent read.
 // In a cluster, one exchange through distributed shared memory then gives the unit's per-head
 // maximum and normaliser: every CTA rewrites its tokens' scores and combines one slice of the
 // G x D outputs from all CTAs' partials. (Exchanging the statistics between the two phases instead
@@ -147,6 +149,10 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         const int rows = min(kStages * kTile, p.C - est_j0);
         if (rows > 0) ptx::prefetch_l2(p.k_cache + (row_base + est_j0) * D, (uint32_t)rows * D * 2);
     }
+    // Launched as a programmatic dependent of the previous kernel on the stream, the CTA may start
+    // before that kernel ends: everything from here on reads what it wrote (lengths, pages,
+    // cache rows, scores, queries), so wait for its completion. (The prefetch above is a hint.)
+    ptx::grid_dependency_wait();
     // Paged: before the length is known, the producer reads the page-table entries of the range the
     // launch's length hint predicts and pulls those tiles into L2 (kept when the prediction holds).
     int est_j0 = -1, est_tiles = 0;
@@ -526,6 +532,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         }
     }
     if (!ok) raise_status(p.status, VOXZIP_DEV_TIMEOUT);
+    ptx::launch_dependents();  // streaming is over: the next launch may begin its prologue
     __syncthreads();
     if (clustered) {
         cluster.sync();  // every CTA's m_cta, z_cta, o_cta are final
@@ -681,14 +688,22 @@ cudaError_t launch_t(const CUtensorMap &tmk, const CUtensorMap &tmv, const MmaPa
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = Layout<K::D, K::NT, K::NS>::bytes(prm.chunk_cap);
     cfg.stream = stream;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = (unsigned)S;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // overlap the previous kernel's tail
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, tmk, tmv, prm);
+    cfg.numAttrs = 2;
+    cudaError_t err = cudaLaunchKernelEx(&cfg, kern, tmk, tmv, prm);
+    if (err == cudaErrorNotSupported || err == cudaErrorInvalidValue) {  // no programmatic launch here
+        cudaGetLastError();
+        cfg.numAttrs = 1;
+        err = cudaLaunchKernelEx(&cfg, kern, tmk, tmv, prm);
+    }
+    return err;
 }
 
 struct Plan {

@@ -28,6 +28,7 @@
 #include "common.cuh"
 #include "evict_policy.cuh"
 #include "paged.cuh"
+#include "ptx.cuh"
 
 namespace voxzip {
 namespace {
@@ -168,6 +169,7 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
 
     const int tid = threadIdx.x;
     const UnitIdx ui = unit_of(blockIdx.x, p.B, p.L, p.Hkv, p.layer_begin);
+    ptx::grid_dependency_wait();  // a programmatic dependent of the previous kernel: wait for its writes
     const int32_t n = p.len[ui.cache_unit];
     const Split sp = split_of(p, ui);
     const int32_t bud = sp.bud, M = sp.M, T_ = sp.T, N = sp.N;
@@ -323,6 +325,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
     __shared__ int resume_at;
     const int tid = threadIdx.x;
     const UnitIdx ui = unit_of(blockIdx.x, p.B, p.L, p.Hkv, p.layer_begin);
+    ptx::grid_dependency_wait();  // a programmatic dependent of the previous kernel: wait for its writes
     const int32_t n = p.len[ui.cache_unit];
     const Split sp = split_of(p, ui);
     const int32_t bud = sp.bud, M = sp.M, T_ = sp.T, N = sp.N;
@@ -455,11 +458,25 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
 
 template <typename T, int D, bool kPaged = false>
 cudaError_t launch_t(const EvictParams &prm, int units, bool fill, cudaStream_t stream) {
-    if (fill)
-        evict_fill_kernel<T, D, kPaged><<<units, kThreads, 0, stream>>>(prm);
-    else
-        evict_kernel<T, D, kPaged><<<units, kThreads, 0, stream>>>(prm);
-    return cudaGetLastError();
+    // A programmatic dependent of the previous kernel (the decode step): the kernels wait for it
+    // before their first read, and a launch without that attribute is the fallback.
+    void (*kern)(EvictParams) = fill ? evict_fill_kernel<T, D, kPaged> : evict_kernel<T, D, kPaged>;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)units, 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t err = cudaLaunchKernelEx(&cfg, kern, prm);
+    if (err == cudaErrorNotSupported || err == cudaErrorInvalidValue) {
+        cudaGetLastError();
+        cfg.numAttrs = 0;
+        err = cudaLaunchKernelEx(&cfg, kern, prm);
+    }
+    return err;
 }
 
 }  // namespace
