@@ -10,8 +10,9 @@
 //               group j = [floor(j*l/g), floor((j+1)*l/g)), Eq. 5 chronological order); the first
 //               token of each slot records the slot's source range and anchor row;
 //   fuse_rows   K/V level, head_dim 64 or 128: one warp-slice per output slot of every (layer,
-//               kv-head) unit: the fp32 mean of the slot's source rows (a copy when the range has
-//               one row) plus the anchor row, rounded once to the cache dtype; K and V in the same
+//               kv-head) unit (a lane owns one 16-byte vector of the row; four source rows in
+//               flight): the fp32 mean of the slot's source rows (a copy when the range has one
+//               row) plus the anchor row, rounded once to the cache dtype; K and V in the same
 //               pass; pos and score = 0;
 //   fuse_wide   embedding level, any width that is a whole number of 16-byte vectors: one warp per
 //               output row of a sequence, the same arithmetic.
@@ -35,6 +36,45 @@ int sm_count() {
         cached[dev] = cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0 ? n : 148;
     }
     return cached[dev];
+}
+
+// acc[e] += element e of a 16-byte vector (4 fp32 or 8 bf16 values, low address first).
+template <typename T>
+__device__ __forceinline__ void accumulate16(float *acc, uint4 x);
+template <>
+__device__ __forceinline__ void accumulate16<float>(float *acc, uint4 x) {
+    acc[0] += __uint_as_float(x.x);
+    acc[1] += __uint_as_float(x.y);
+    acc[2] += __uint_as_float(x.z);
+    acc[3] += __uint_as_float(x.w);
+}
+template <>
+__device__ __forceinline__ void accumulate16<__nv_bfloat16>(float *acc, uint4 x) {
+    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        acc[2 * i] += __uint_as_float(w[i] << 16);
+        acc[2 * i + 1] += __uint_as_float(w[i] & 0xffff0000u);
+    }
+}
+// The 16-byte vector of acc rounded to T (round to nearest even).
+template <typename T>
+__device__ __forceinline__ uint4 pack16(const float *acc);
+template <>
+__device__ __forceinline__ uint4 pack16<float>(const float *acc) {
+    return make_uint4(__float_as_uint(acc[0]), __float_as_uint(acc[1]), __float_as_uint(acc[2]),
+                      __float_as_uint(acc[3]));
+}
+template <>
+__device__ __forceinline__ uint4 pack16<__nv_bfloat16>(const float *acc) {
+    uint32_t w[4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * i]));
+        const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * i + 1]));
+        w[i] = lo | (hi << 16);
+    }
+    return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
 constexpr int kScanThreads = 512;
@@ -239,8 +279,10 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
                  const T *__restrict__ anchor_k, const T *__restrict__ anchor_v, FuseWorkspace ws,
                  T *__restrict__ k_cache, T *__restrict__ v_cache, float *__restrict__ score,
                  int32_t *__restrict__ pos, int32_t *__restrict__ len, PageView pv) {
-    constexpr int kLanesPerRow = D / 4;          // each lane owns 4 consecutive elements
+    constexpr int kElems = 16 / (int)sizeof(T);  // each lane owns one 16-byte vector of a row
+    constexpr int kLanesPerRow = D / kElems;
     constexpr int kRowsPerWarp = 32 / kLanesPerRow;
+    constexpr int kRowVecs = D / kElems;          // 16-byte vectors per row
     const int u = blockIdx.y;                    // cache unit (b, l, h)
     const int b = u / (L * Hkv);
     int32_t out_len = ws.seq_len[b];
@@ -248,10 +290,12 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
     if (blockIdx.x == 0 && threadIdx.x == 0) len[u] = out_len < 0 ? 0 : out_len;
     if (out_len < 0) return;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int sub = lane / kLanesPerRow, e = (lane % kLanesPerRow) * 4;
+    const int sub = lane / kLanesPerRow, e = (lane % kLanesPerRow) * kElems;
     const int64_t in_base = (int64_t)u * stride * D;
     const int64_t out_base = kPaged ? 0 : (int64_t)u * C * D;
     const int64_t anc_base = (int64_t)u * anchor_stride * D;
+    const uint4 *kin = reinterpret_cast<const uint4 *>(k_prefill + in_base + e);  // vector e of row 0
+    const uint4 *vin = reinterpret_cast<const uint4 *>(v_prefill + in_base + e);
     const int32_t *src = ws.slot_src + (int64_t)b * stride;
     const int32_t *send = ws.slot_end + (int64_t)b * stride;
     const int32_t *anc = ws.slot_anchor + (int64_t)b * stride;
@@ -262,32 +306,51 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
         const int s = slot0 + k * kRowsPerWarp + sub;
         if (s >= out_len) break;
         const int32_t r0 = src[s], r1 = send[s];
-        float4 sk = make_float4(0.f, 0.f, 0.f, 0.f), sv = sk;
-        for (int32_t r = r0; r < r1; ++r) {
-            const float4 a = load4(k_prefill + in_base + (int64_t)r * D + e);
-            const float4 c = load4(v_prefill + in_base + (int64_t)r * D + e);
-            sk.x += a.x; sk.y += a.y; sk.z += a.z; sk.w += a.w;
-            sv.x += c.x; sv.y += c.y; sv.z += c.z; sv.w += c.w;
+        float sk[kElems], sv[kElems];
+#pragma unroll
+        for (int i = 0; i < kElems; ++i) sk[i] = sv[i] = 0.f;
+        int32_t r = r0;
+        for (; r + 4 <= r1; r += 4) {  // four rows' loads in flight, then their sums in token order
+            uint4 xk[4], xv[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                xk[i] = __ldcs(kin + (int64_t)(r + i) * kRowVecs);
+                xv[i] = __ldcs(vin + (int64_t)(r + i) * kRowVecs);
+            }
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                accumulate16<T>(sk, xk[i]);
+                accumulate16<T>(sv, xv[i]);
+            }
+        }
+        for (; r < r1; ++r) {
+            accumulate16<T>(sk, __ldcs(kin + (int64_t)r * kRowVecs));
+            accumulate16<T>(sv, __ldcs(vin + (int64_t)r * kRowVecs));
         }
         if (r1 - r0 > 1) {
             const float cnt = (float)(r1 - r0);
-            sk.x = __fdiv_rn(sk.x, cnt); sk.y = __fdiv_rn(sk.y, cnt);
-            sk.z = __fdiv_rn(sk.z, cnt); sk.w = __fdiv_rn(sk.w, cnt);
-            sv.x = __fdiv_rn(sv.x, cnt); sv.y = __fdiv_rn(sv.y, cnt);
-            sv.z = __fdiv_rn(sv.z, cnt); sv.w = __fdiv_rn(sv.w, cnt);
+#pragma unroll
+            for (int i = 0; i < kElems; ++i) {
+                sk[i] = __fdiv_rn(sk[i], cnt);
+                sv[i] = __fdiv_rn(sv[i], cnt);
+            }
         }
         const int32_t a_row = anc[s];
         if (anchor_k != nullptr && a_row >= 0) {
-            const float4 ak = load4(anchor_k + anc_base + (int64_t)a_row * D + e);
-            const float4 av = load4(anchor_v + anc_base + (int64_t)a_row * D + e);
-            sk.x = __fadd_rn(sk.x, ak.x); sk.y = __fadd_rn(sk.y, ak.y);
-            sk.z = __fadd_rn(sk.z, ak.z); sk.w = __fadd_rn(sk.w, ak.w);
-            sv.x = __fadd_rn(sv.x, av.x); sv.y = __fadd_rn(sv.y, av.y);
-            sv.z = __fadd_rn(sv.z, av.z); sv.w = __fadd_rn(sv.w, av.w);
+            float ak[kElems], av[kElems];
+#pragma unroll
+            for (int i = 0; i < kElems; ++i) ak[i] = av[i] = 0.f;
+            accumulate16<T>(ak, *reinterpret_cast<const uint4 *>(anchor_k + anc_base + (int64_t)a_row * D + e));
+            accumulate16<T>(av, *reinterpret_cast<const uint4 *>(anchor_v + anc_base + (int64_t)a_row * D + e));
+#pragma unroll
+            for (int i = 0; i < kElems; ++i) {
+                sk[i] = __fadd_rn(sk[i], ak[i]);
+                sv[i] = __fadd_rn(sv[i], av[i]);
+            }
         }
         const int64_t orow = kPaged ? paged_row(pv, u, s) : s;
-        store4(k_cache + out_base + orow * D + e, sk);
-        store4(v_cache + out_base + orow * D + e, sv);
+        *reinterpret_cast<uint4 *>(k_cache + out_base + orow * D + e) = pack16<T>(sk);
+        *reinterpret_cast<uint4 *>(v_cache + out_base + orow * D + e) = pack16<T>(sv);
         if (e == 0) {
             pos[(int64_t)u * C + s] = r0;
             score[(int64_t)u * C + s] = 0.f;
@@ -300,7 +363,7 @@ cudaError_t launch_fuse_rows(const voxzip_cache_desc &d, int32_t stride, int32_t
                              const void *kp, const void *vp, const void *ak, const void *av,
                              const FuseWorkspace &ws, void *kc, void *vc, float *score, int32_t *pos,
                              int32_t *len, cudaStream_t stream, PageView pv = PageView{nullptr, nullptr, nullptr, 0}) {
-    constexpr int kRowsPerWarp = 32 / (D / 4);
+    constexpr int kRowsPerWarp = 32 / (D * (int)sizeof(T) / 16);  // as in the kernel
     const int slots_per_block = kFuseWarps * kSlotsPerWarp * kRowsPerWarp;
     const int64_t units = (int64_t)d.batch * d.layers * d.kv_heads;
     // A grid-stride loop over each unit's output slots: about six CTAs per SM in all, never more
@@ -316,45 +379,6 @@ cudaError_t launch_fuse_rows(const voxzip_cache_desc &d, int32_t stride, int32_t
 }
 
 constexpr int kWideWarps = 8;
-
-// acc[e] += element e of a 16-byte vector (4 fp32 or 8 bf16 values, low address first).
-template <typename T>
-__device__ __forceinline__ void accumulate16(float *acc, uint4 x);
-template <>
-__device__ __forceinline__ void accumulate16<float>(float *acc, uint4 x) {
-    acc[0] += __uint_as_float(x.x);
-    acc[1] += __uint_as_float(x.y);
-    acc[2] += __uint_as_float(x.z);
-    acc[3] += __uint_as_float(x.w);
-}
-template <>
-__device__ __forceinline__ void accumulate16<__nv_bfloat16>(float *acc, uint4 x) {
-    const uint32_t w[4] = {x.x, x.y, x.z, x.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        acc[2 * i] += __uint_as_float(w[i] << 16);
-        acc[2 * i + 1] += __uint_as_float(w[i] & 0xffff0000u);
-    }
-}
-// The 16-byte vector of acc rounded to T (round to nearest even).
-template <typename T>
-__device__ __forceinline__ uint4 pack16(const float *acc);
-template <>
-__device__ __forceinline__ uint4 pack16<float>(const float *acc) {
-    return make_uint4(__float_as_uint(acc[0]), __float_as_uint(acc[1]), __float_as_uint(acc[2]),
-                      __float_as_uint(acc[3]));
-}
-template <>
-__device__ __forceinline__ uint4 pack16<__nv_bfloat16>(const float *acc) {
-    uint32_t w[4];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const uint32_t lo = __bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * i]));
-        const uint32_t hi = __bfloat16_as_ushort(__float2bfloat16_rn(acc[2 * i + 1]));
-        w[i] = lo | (hi << 16);
-    }
-    return make_uint4(w[0], w[1], w[2], w[3]);
-}
 
 // Embedding-level fusion: one warp per output row of sequence b; each lane owns 16-byte vectors
 // v and v + 32 of the row (two in flight per source row). The arithmetic is fuse_rows' (fp32 sum
