@@ -350,15 +350,28 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
         valid = true;
         return (uint32_t)ps[j];
     };
+    // The bits any position sets: radix passes over high digits that are zero in every position
+    // (positions below 2^16, say) decide nothing and are skipped.
+    uint32_t any = 0u;
+    for (int j = tid; j < n; j += kThreads) any |= (uint32_t)ps[j];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) any |= __shfl_xor_sync(0xffffffffu, any, o);
+    if ((tid & 31) == 0) warp_sums[tid >> 5] = (int)any;
+    __syncthreads();
+    any = 0u;
+#pragma unroll
+    for (int w = 0; w < kThreads / 32; ++w) any |= (uint32_t)warp_sums[w];
+    __syncthreads();
+    const int top_shift = any >> 24 ? 24 : any >> 16 ? 16 : any >> 8 ? 8 : 0;
     uint32_t p_lo = 0u, p_hi = 0xffffffffu;
     if (T_ > 0) {
         RadixState st{0u, T_, 0};
-        for (int shift = 24; shift >= 0; shift -= 8) radix_pass<false>(shift, 0, n, pkey, st, hist, &shared_st);
+        for (int shift = top_shift; shift >= 0; shift -= 8) radix_pass<false>(shift, 0, n, pkey, st, hist, &shared_st);
         p_lo = st.prefix;
     }
     if (M > 0) {
         RadixState st{0u, M, 0};
-        for (int shift = 24; shift >= 0; shift -= 8) radix_pass<true>(shift, 0, n, pkey, st, hist, &shared_st);
+        for (int shift = top_shift; shift >= 0; shift -= 8) radix_pass<true>(shift, 0, n, pkey, st, hist, &shared_st);
         p_hi = st.prefix;
     }
     auto middle = [&](uint32_t q) { return !(T_ > 0 && q <= p_lo) && !(M > 0 && q >= p_hi); };
@@ -382,7 +395,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
                 valid = middle(q) && score_key(sc[j]) == thr;
                 return q;
             };
-            for (int shift = 24; shift >= 0; shift -= 8)
+            for (int shift = top_shift; shift >= 0; shift -= 8)
                 radix_pass<false>(shift, 0, n, tkey, sq, hist, &shared_st);
             pos_thr = sq.prefix;
         }
