@@ -621,11 +621,16 @@ def cpu_sample(w, n_units=0, inputs=None, compaction="ordered"):
         list(ex.map(one, args))
     wall = time.perf_counter() - t0
     full = wall * w.units / len(units)
+    t1 = time.perf_counter()
+    one(args[0])                      # one unit alone: the single-thread rate
+    one_unit = time.perf_counter() - t1
     return {"value": round(w.steps / full, 4), "unit": UNIT, "cores": used, "kind": "oracle",
             "sample": (f"{len(units)} of {w.units} units (seeded choice), each through the whole request "
                        f"({w.steps} decode steps, evictions every {w.interval}); {wall:.1f} s wall on {used} "
                        f"threads, scaled by {w.units}/{len(units)} to the whole workload"),
-            "sample_wall_s": round(wall, 2)}, inputs
+            "sample_wall_s": round(wall, 2),
+            "single_thread_value": round(w.steps / (one_unit * w.units), 5),
+            "single_thread_sample": f"one unit alone, {one_unit:.1f} s, scaled by {w.units} units"}, inputs
 
 
 def reference_arm(args, rank, world):
