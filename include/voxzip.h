@@ -63,6 +63,8 @@ typedef enum {
                                       are not valid (never expected; reported instead of hanging) */
 #define VOXZIP_DEV_BAD_POSITIONS 0x20u /* a unit's positions were not unique, so a hole-filling
                                           eviction could not keep exactly `budget` rows */
+#define VOXZIP_DEV_BOUNDS 0x40u    /* checked builds only (-DVOXZIP_CHECKED): an index a kernel was
+                                      about to use fell outside its buffer; the access was skipped */
 
 typedef enum { VOXZIP_F32 = 0, VOXZIP_BF16 = 1 } voxzip_dtype;
 
@@ -368,6 +370,15 @@ voxzip_status voxzip_evict_paged(const voxzip_cache_desc *desc, const voxzip_pag
  * (VOXZIP_DEV_* flags accumulated by earlier calls) and clears it.
  */
 voxzip_status voxzip_get_status(uint32_t *bits, voxzip_stream_t stream);
+
+/*
+ * Self-test of the bounded waits: failure detection exercised without a GPU fault. One CTA arms an
+ * mbarrier for 16 bytes that never arrive and waits on it with the bounded wait the decode kernel
+ * uses on its TMA ring, giving up after `limit` polls (1 to 2^20). The give-up sets
+ * VOXZIP_DEV_TIMEOUT in the status word, as a decode whose loads never landed would. No copy is
+ * issued, so nothing can fault. Asynchronous on `stream`; VOXZIP_EINVAL for a limit out of range.
+ */
+voxzip_status voxzip_selftest_bounded_wait(uint32_t limit, voxzip_stream_t stream);
 
 /* Human-readable name of a status code (static storage). */
 const char *voxzip_status_string(voxzip_status status);

@@ -13,11 +13,16 @@ from dataclasses import dataclass
 
 import torch
 
-from .build import LIB_PATH
+from .build import CHECKED_LIB_PATH
+from .build import LIB_PATH as _REGULAR_LIB_PATH
+
+# VOXZIP_CHECKED=1 selects the range-checked build (kernels report out-of-range accesses as
+# DEV_BOUNDS instead of making them); it is slower and meant for tests.
+LIB_PATH = CHECKED_LIB_PATH if os.environ.get("VOXZIP_CHECKED", "0") not in ("", "0") else _REGULAR_LIB_PATH
 
 VOXZIP_OK, VOXZIP_EINVAL, VOXZIP_EUNSUPPORTED, VOXZIP_ECUDA, VOXZIP_ESCRATCH = 0, 1, 2, 3, 4
 DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_BAD_BUDGET, DEV_TIMEOUT = 0x1, 0x2, 0x4, 0x8, 0x10
-DEV_BAD_POSITIONS = 0x20
+DEV_BAD_POSITIONS, DEV_BOUNDS = 0x20, 0x40
 VOXZIP_COMPACT_ORDERED, VOXZIP_COMPACT_FILL = 0, 1
 VOXZIP_F32, VOXZIP_BF16 = 0, 1
 
@@ -129,6 +134,8 @@ def lib() -> ctypes.CDLL:
                                                    _f32, _i32, _vp, _vp]
             L.voxzip_evict_paged.argtypes = [_DP, _PP, _i32, _i32, _vp, _vp, _vp, _vp, ctypes.POINTER(_EvictPolicy),
                                              _vp]
+            L.voxzip_selftest_bounded_wait.argtypes = [ctypes.c_uint32, _vp]
+            L.voxzip_selftest_bounded_wait.restype = _i32
             L.voxzip_segments_to_spans.argtypes = [_i32, _vp, _vp, _vp, _vp, _f64, _i32, _i32, _f64, _vp, _vp, _vp,
                                                    _vp, _vp]
             L.voxzip_embed_fuse.argtypes = [_EP, _vp, _i32, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _i32,
@@ -504,6 +511,12 @@ def voxzip_evict_ex(desc: CacheDesc, layer_begin: int, layer_count: int, k_cache
     _check("voxzip_evict_ex", lib().voxzip_evict_ex(
         ctypes.byref(d), int(layer_begin), int(layer_count), _ptr(k_cache), _ptr(v_cache), _ptr(score), _ptr(pos),
         _ptr(len_), _ptr(budget), ctypes.byref(pol), _stream(stream)))
+
+
+def voxzip_selftest_bounded_wait(limit: int = 1000, stream=None) -> None:
+    """Launches the bounded-wait self-test: a wait that can never complete gives up after `limit`
+    polls and sets DEV_TIMEOUT in the status word (read it with voxzip_get_status)."""
+    _check("voxzip_selftest_bounded_wait", lib().voxzip_selftest_bounded_wait(int(limit), _stream(stream)))
 
 
 def voxzip_get_status(stream=None) -> int:

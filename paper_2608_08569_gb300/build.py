@@ -2,6 +2,11 @@
 
 Each ``csrc/*.cu`` file compiles to an object in ``_build/`` in parallel, then nvcc links the
 shared library next to this file. ``python -m paper_2608_08569_gb300.build`` runs it.
+
+``--checked`` builds ``libvoxzip_checked.so`` instead, with ``-DVOXZIP_CHECKED``: its kernels
+range-check the indices of their global accesses, skip an access that is out of range and set
+``VOXZIP_DEV_BOUNDS`` in the status word. Setting ``VOXZIP_CHECKED=1`` in the environment makes
+the binding load that library.
 """
 from __future__ import annotations
 
@@ -17,6 +22,7 @@ ROOT = os.path.dirname(PKG_DIR)
 CSRC = os.path.join(PKG_DIR, "csrc")
 BUILD_DIR = os.path.join(ROOT, "_build")
 LIB_PATH = os.path.join(PKG_DIR, "libvoxzip.so")
+CHECKED_LIB_PATH = os.path.join(PKG_DIR, "libvoxzip_checked.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "-cudart", "shared",
               "--expt-relaxed-constexpr", "-Xptxas", "-v", "-I" + os.path.join(ROOT, "include")]
@@ -38,24 +44,29 @@ def _deps():
         os.path.join(ROOT, "include", "voxzip.h")]
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB_PATH):
+def up_to_date(checked: bool = False) -> bool:
+    lib_path = CHECKED_LIB_PATH if checked else LIB_PATH
+    if not os.path.exists(lib_path):
         return False
-    t = os.path.getmtime(LIB_PATH)
+    t = os.path.getmtime(lib_path)
     return all(os.path.getmtime(p) <= t for p in _deps())
 
 
-def build_library(force: bool = False, verbose: bool = False) -> str:
-    """Compile and link ``libvoxzip.so``; returns its path. Skips work when up to date."""
-    if not force and up_to_date():
-        return LIB_PATH
+def build_library(force: bool = False, verbose: bool = False, checked: bool = False) -> str:
+    """Compile and link ``libvoxzip.so`` (``libvoxzip_checked.so`` with `checked`); returns its
+    path. Skips work when up to date."""
+    lib_path = CHECKED_LIB_PATH if checked else LIB_PATH
+    if not force and up_to_date(checked):
+        return lib_path
     nvcc = _nvcc()
-    os.makedirs(BUILD_DIR, exist_ok=True)
+    build_dir = os.path.join(BUILD_DIR, "checked") if checked else BUILD_DIR
+    os.makedirs(build_dir, exist_ok=True)
     srcs = _sources()
+    flags = NVCC_FLAGS + (["-DVOXZIP_CHECKED"] if checked else [])
 
     def compile_one(src):
-        obj = os.path.join(BUILD_DIR, os.path.basename(src)[:-3] + ".o")
-        cmd = [nvcc, *ARCH, *NVCC_FLAGS, "-c", src, "-o", obj]
+        obj = os.path.join(build_dir, os.path.basename(src)[:-3] + ".o")
+        cmd = [nvcc, *ARCH, *flags, "-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed on {src}:\n{r.stdout}\n{r.stderr}")
@@ -65,19 +76,19 @@ def build_library(force: bool = False, verbose: bool = False) -> str:
 
     with cf.ThreadPoolExecutor(max_workers=max(1, min(len(srcs), os.cpu_count() or 1))) as ex:
         objs = list(ex.map(compile_one, srcs))
-    tmp = LIB_PATH + f".tmp{os.getpid()}"
+    tmp = lib_path + f".tmp{os.getpid()}"
     cmd = [nvcc, *ARCH, "-shared", "-cudart", "shared", "-Xlinker", "-rpath,/usr/local/cuda/lib64", "-o", tmp,
            *objs]
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"nvcc link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB_PATH)
+    os.replace(tmp, lib_path)
     if verbose:
         for o in objs:
             with open(o + ".ptxas.txt") as f:
                 sys.stdout.write(f.read())
-    return LIB_PATH
+    return lib_path
 
 
 if __name__ == "__main__":
-    print(build_library(force="--force" in sys.argv, verbose="-v" in sys.argv))
+    print(build_library(force="--force" in sys.argv, verbose="-v" in sys.argv, checked="--checked" in sys.argv))

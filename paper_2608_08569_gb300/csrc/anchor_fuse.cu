@@ -91,6 +91,7 @@ struct FuseWorkspace {
     int32_t *slot_src;       // [B][stride] first prompt token of each slot
     int32_t *slot_end;       // [B][stride] one past the last prompt token of each slot
     int32_t *slot_anchor;    // [B][stride] anchor row of each slot, -1 for copied rows
+    int32_t *status;         // the call's device status word (not part of the workspace bytes)
 };
 
 __host__ __device__ inline size_t align256(size_t x) { return (x + 255) & ~size_t(255); }
@@ -306,6 +307,7 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
         const int s = slot0 + k * kRowsPerWarp + sub;
         if (s >= out_len) break;
         const int32_t r0 = src[s], r1 = send[s];
+        if (!VOXZIP_IN_RANGE(ws.status, r0 >= 0 && r0 < r1 && r1 <= stride && s < C)) continue;
         float sk[kElems], sv[kElems];
 #pragma unroll
         for (int i = 0; i < kElems; ++i) sk[i] = sv[i] = 0.f;
@@ -336,7 +338,7 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
             }
         }
         const int32_t a_row = anc[s];
-        if (anchor_k != nullptr && a_row >= 0) {
+        if (anchor_k != nullptr && a_row >= 0 && VOXZIP_IN_RANGE(ws.status, a_row < anchor_stride)) {
             float ak[kElems], av[kElems];
 #pragma unroll
             for (int i = 0; i < kElems; ++i) ak[i] = av[i] = 0.f;
@@ -403,6 +405,9 @@ fuse_wide_kernel(int32_t C, int32_t stride, int32_t D, int32_t text_stride, cons
     const int32_t *anc = ws.slot_anchor + (int64_t)b * stride;
     for (int s = blockIdx.x * kWideWarps + warp; s < out_len; s += gridDim.x * kWideWarps) {
         const int32_t r0 = src[s], r1 = send[s], a_row = anc[s];
+        if (!VOXZIP_IN_RANGE(ws.status, r0 >= 0 && r0 < r1 && r1 <= stride && s < C &&
+                                         (txt == nullptr || a_row < text_stride)))
+            continue;
         const float cnt = (float)(r1 - r0);
         for (int v0 = lane; v0 < vecs; v0 += 64) {
             const bool two = v0 + 32 < vecs;
@@ -518,6 +523,7 @@ cudaError_t launch_anchor_fuse(const voxzip_cache_desc &d, const void *k_prefill
                                int32_t *status, cudaStream_t stream) {
     FuseWorkspace ws;
     carve(d, prefill_stride, num_spans, static_cast<char *>(workspace), &ws);
+    ws.status = status;
     cudaError_t err = launch_slot_plan(d.batch, d.capacity, prefill_stride, num_spans, anchor_stride,
                                        anchor_k != nullptr, true, in_len, audio_begin, audio_len, span_off,
                                        span_start, span_end, span_groups, ws, slot_map, status, stream);
@@ -550,6 +556,7 @@ cudaError_t launch_anchor_fuse_paged(const voxzip_cache_desc &d, const voxzip_pa
                                      int32_t *slot_map, void *workspace, int32_t *status, cudaStream_t stream) {
     FuseWorkspace ws;
     carve(d, prefill_stride, num_spans, static_cast<char *>(workspace), &ws);
+    ws.status = status;
     const PageView pv{pc.page_table, pc.free_pages, pc.free_count, pc.max_pages};
     const int64_t units = (int64_t)d.batch * d.layers * d.kv_heads;
     const unsigned blocks = (unsigned)((units + 7) / 8);
@@ -614,6 +621,7 @@ cudaError_t launch_embed_fuse(int32_t B, int32_t D, int32_t C, bool bf16, const 
     d.batch = B;
     FuseWorkspace ws;
     carve(d, stride, num_spans, static_cast<char *>(workspace), &ws);
+    ws.status = status;
     cudaError_t err = launch_slot_plan(B, C, stride, num_spans, text_stride, e_text != nullptr, keep_background,
                                        in_len, audio_begin, audio_len, span_off, span_start, span_end, span_groups,
                                        ws, slot_map, status, stream);

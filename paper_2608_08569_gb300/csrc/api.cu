@@ -1,11 +1,14 @@
 // C ABI of the VoxZip library (declared in include/voxzip.h): argument validation, the device
-// status word, and dispatch to the kernel launchers. Nothing here allocates device memory.
+// status word, and dispatch to the kernel launchers. Nothing here allocates device memory. Every
+// entry point opens an NVTX range of its own name (a no-op unless a profiler listens).
 #include <math.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include "common.cuh"
 #include "embed.cuh"
 #include "evict_policy.cuh"
 #include "paged.cuh"
+#include "ptx.cuh"
 
 namespace {
 
@@ -46,6 +49,23 @@ voxzip_status from_cuda(cudaError_t e) { return e == cudaSuccess ? VOXZIP_OK : V
 
 constexpr int kMaxGridY = 65535;
 
+// An NVTX range for the lifetime of an entry point.
+struct Range {
+    explicit Range(const char *name) { nvtxRangePushA(name); }
+    ~Range() { nvtxRangePop(); }
+};
+
+// One CTA: an mbarrier armed for 16 bytes that never arrive, waited on with the bounded wait.
+__global__ void selftest_wait_kernel(uint32_t limit, int32_t *status) {
+    __shared__ uint64_t bar;
+    if (threadIdx.x == 0) {
+        voxzip::ptx::mbar_init(&bar, 1);
+        voxzip::ptx::fence_mbar_init();
+        voxzip::ptx::mbar_arrive_expect_tx(&bar, 16);
+        if (!voxzip::ptx::mbar_wait_bounded(&bar, 0, limit)) voxzip::raise_status(status, VOXZIP_DEV_TIMEOUT);
+    }
+}
+
 }  // namespace
 
 // The status word's device address on the current device, for entry points in other files.
@@ -68,6 +88,7 @@ const char *voxzip_status_string(voxzip_status s) {
 
 size_t voxzip_anchor_fuse_workspace_size(const voxzip_cache_desc *desc, int32_t prefill_stride,
                                          int32_t num_spans) {
+    Range range("voxzip_anchor_fuse_workspace_size");
     if (!desc_ok(desc) || prefill_stride < 1 || num_spans < 0) return 0;
     return voxzip::anchor_fuse_workspace_bytes(*desc, prefill_stride, num_spans);
 }
@@ -82,6 +103,7 @@ voxzip_status voxzip_anchor_fuse(const voxzip_cache_desc *desc, const void *k_pr
                                  void *k_cache, void *v_cache, float *score, int32_t *pos,
                                  int32_t *len, int32_t *slot_map, void *workspace,
                                  size_t workspace_bytes, voxzip_stream_t stream) {
+    Range range("voxzip_anchor_fuse");
     if (!desc_ok(desc) || prefill_stride < 1 || num_spans < 0) return VOXZIP_EINVAL;
     if (!k_prefill || !v_prefill || !in_len || !audio_begin || !audio_len || !span_off || !k_cache ||
         !v_cache || !score || !pos || !len || !workspace)
@@ -126,12 +148,14 @@ bool policy_ok(const voxzip_evict_policy &p) {
 
 voxzip_status voxzip_paged_init(const voxzip_cache_desc *desc, const voxzip_paged_cache *paged, int32_t *len,
                                 voxzip_stream_t stream) {
+    Range range("voxzip_paged_init");
     if (!paged_ok(desc, paged) || !len) return VOXZIP_EINVAL;
     return from_cuda(voxzip::launch_paged_init(*desc, *paged, len, reinterpret_cast<cudaStream_t>(stream)));
 }
 
 size_t voxzip_anchor_fuse_paged_workspace_size(const voxzip_cache_desc *desc, int32_t prefill_stride,
                                                int32_t num_spans) {
+    Range range("voxzip_anchor_fuse_paged_workspace_size");
     if (!desc_ok(desc) || prefill_stride < 1 || num_spans < 0) return 0;
     return voxzip::anchor_fuse_paged_workspace_bytes(*desc, prefill_stride, num_spans);
 }
@@ -146,6 +170,7 @@ voxzip_status voxzip_anchor_fuse_paged(const voxzip_cache_desc *desc, const voxz
                                        const void *anchor_v, int32_t anchor_stride, float *score,
                                        int32_t *pos, int32_t *len, int32_t *slot_map, void *workspace,
                                        size_t workspace_bytes, voxzip_stream_t stream) {
+    Range range("voxzip_anchor_fuse_paged");
     if (!paged_ok(desc, paged) || prefill_stride < 1 || num_spans < 0) return VOXZIP_EINVAL;
     if (!k_prefill || !v_prefill || !in_len || !audio_begin || !audio_len || !span_off || !score || !pos || !len ||
         !workspace)
@@ -175,6 +200,7 @@ voxzip_status voxzip_decode_step_paged(const voxzip_cache_desc *desc, const voxz
                                        float *score, int32_t *pos, int32_t *len, float gamma,
                                        float sm_scale, int32_t max_len, void *out,
                                        voxzip_stream_t stream) {
+    Range range("voxzip_decode_step_paged");
     if (!paged_ok(desc, paged)) return VOXZIP_EINVAL;
     if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
         return VOXZIP_EINVAL;
@@ -198,6 +224,7 @@ voxzip_status voxzip_evict_paged(const voxzip_cache_desc *desc, const voxzip_pag
                                  int32_t layer_begin, int32_t layer_count, float *score, int32_t *pos,
                                  int32_t *len, const int32_t *budget, const voxzip_evict_policy *policy,
                                  voxzip_stream_t stream) {
+    Range range("voxzip_evict_paged");
     if (!paged_ok(desc, paged) || policy == nullptr || !policy_ok(*policy)) return VOXZIP_EINVAL;
     if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
         return VOXZIP_EINVAL;
@@ -216,6 +243,7 @@ voxzip_status voxzip_segments_to_spans(int32_t n, const double *t_start, const d
                                        double threshold, int32_t *span_start, int32_t *span_end,
                                        int32_t *span_groups, int32_t *seg_index,
                                        int32_t *num_spans) {
+    Range range("voxzip_segments_to_spans");
     if (n < 0 || !num_spans || !(tau_total > 0.0) || isinf(tau_total) || audio_len < 0 || audio_begin < 0 ||
         (int64_t)audio_begin + audio_len > INT32_MAX)
         return VOXZIP_EINVAL;
@@ -259,6 +287,7 @@ bool embed_desc_ok(const voxzip_embed_desc *d) {
 }  // namespace
 
 size_t voxzip_embed_fuse_workspace_size(const voxzip_embed_desc *desc, int32_t stride, int32_t num_spans) {
+    Range range("voxzip_embed_fuse_workspace_size");
     if (!embed_desc_ok(desc) || stride < 1 || num_spans < 0) return 0;
     return voxzip::embed_fuse_workspace_bytes(desc->batch, stride, num_spans);
 }
@@ -271,6 +300,7 @@ voxzip_status voxzip_embed_fuse(const voxzip_embed_desc *desc, const void *e_in,
                                 const void *e_text, int32_t text_stride, int32_t keep_background,
                                 void *e_out, int32_t *pos, int32_t *len, int32_t *slot_map,
                                 void *workspace, size_t workspace_bytes, voxzip_stream_t stream) {
+    Range range("voxzip_embed_fuse");
     if (!embed_desc_ok(desc) || stride < 1 || num_spans < 0) return VOXZIP_EINVAL;
     if (!e_in || !in_len || !audio_begin || !audio_len || !span_off || !e_out || !pos || !len || !workspace)
         return VOXZIP_EINVAL;
@@ -297,6 +327,7 @@ voxzip_status voxzip_decode_step(const voxzip_cache_desc *desc, int32_t layer_be
                                  void *v_cache, float *score, int32_t *pos, int32_t *len,
                                  float gamma, float sm_scale, int32_t max_len, void *out,
                                  voxzip_stream_t stream) {
+    Range range("voxzip_decode_step");
     if (!desc_ok(desc)) return VOXZIP_EINVAL;
     if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
         return VOXZIP_EINVAL;
@@ -323,6 +354,7 @@ voxzip_status voxzip_evict(const voxzip_cache_desc *desc, int32_t layer_begin,
                            int32_t layer_count, void *k_cache, void *v_cache, float *score,
                            int32_t *pos, int32_t *len, const int32_t *budget, int32_t sink,
                            float recent_frac, voxzip_stream_t stream) {
+    Range range("voxzip_evict");
     if (!desc_ok(desc)) return VOXZIP_EINVAL;
     if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
         return VOXZIP_EINVAL;
@@ -342,6 +374,7 @@ voxzip_status voxzip_evict_ex(const voxzip_cache_desc *desc, int32_t layer_begin
                               int32_t layer_count, void *k_cache, void *v_cache, float *score,
                               int32_t *pos, int32_t *len, const int32_t *budget,
                               const voxzip_evict_policy *policy, voxzip_stream_t stream) {
+    Range range("voxzip_evict_ex");
     if (!desc_ok(desc) || policy == nullptr) return VOXZIP_EINVAL;
     if (layer_begin < 0 || layer_count < 1 || layer_begin + (int64_t)layer_count > desc->layers)
         return VOXZIP_EINVAL;
@@ -360,6 +393,7 @@ voxzip_status voxzip_evict_ex(const voxzip_cache_desc *desc, int32_t layer_begin
 }
 
 voxzip_status voxzip_get_status(uint32_t *bits, voxzip_stream_t stream) {
+    Range range("voxzip_get_status");
     if (!bits) return VOXZIP_EINVAL;
     int32_t *status = nullptr;
     voxzip_status st = status_word(&status);
@@ -376,3 +410,13 @@ voxzip_status voxzip_get_status(uint32_t *bits, voxzip_stream_t stream) {
 }
 
 }  // extern "C"
+
+extern "C" voxzip_status voxzip_selftest_bounded_wait(uint32_t limit, voxzip_stream_t stream) {
+    Range range("voxzip_selftest_bounded_wait");
+    if (limit < 1 || limit > (1u << 20)) return VOXZIP_EINVAL;
+    int32_t *status = nullptr;
+    voxzip_status st = status_word(&status);
+    if (st != VOXZIP_OK) return st;
+    selftest_wait_kernel<<<1, 32, 0, reinterpret_cast<cudaStream_t>(stream)>>>(limit, status);
+    return from_cuda(cudaGetLastError());
+}

@@ -49,6 +49,15 @@ __device__ __forceinline__ void raise_status(int32_t *status, uint32_t bits) {
     atomicOr(reinterpret_cast<unsigned int *>(status), bits);
 }
 
+// Builds with -DVOXZIP_CHECKED range-check the indices of the accesses this guards: a violation
+// sets VOXZIP_DEV_BOUNDS and the guarded access is skipped (never a trap). Regular builds compile
+// the checks out.
+#ifdef VOXZIP_CHECKED
+#define VOXZIP_IN_RANGE(status, cond) ((cond) ? true : (voxzip::raise_status((status), VOXZIP_DEV_BOUNDS), false))
+#else
+#define VOXZIP_IN_RANGE(status, cond) true
+#endif
+
 // Unit index helpers. Units of a call are ordered (layer_local, b, h) to match the per-layer
 // activation layout [layer][B][heads][D]; cache arrays are ordered (b, layer, h).
 struct UnitIdx {

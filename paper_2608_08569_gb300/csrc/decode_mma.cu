@@ -75,6 +75,7 @@ struct MmaParams {
     __nv_bfloat16 *out;
     int32_t *status;
     int32_t B, L, Hq, Hkv, G, C, layer_begin, chunk_cap, n_hint;
+    int64_t rows;  // K / V rows the tensor maps cover (the cache, or the page pools)
     float gamma, scale_log2;
     PageView pv;  // paged instantiations: the pools are k_cache / v_cache
 };
@@ -227,10 +228,11 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
         const int64_t src = (act_row * p.Hkv + ui.h) * D + lane * 8;
         kn4 = *reinterpret_cast<const uint4 *>(p.k_new + src);
         vn4 = *reinterpret_cast<const uint4 *>(p.v_new + src);
-        const int64_t dst = (kPaged ? (int64_t)page_new * kPageTokens + (n_old & (kPageTokens - 1)) : row_base + n - 1) * D +
-                            lane * 8;
-        *reinterpret_cast<uint4 *>(p.k_cache + dst) = kn4;
-        *reinterpret_cast<uint4 *>(p.v_cache + dst) = vn4;
+        const int64_t drow = kPaged ? (int64_t)page_new * kPageTokens + (n_old & (kPageTokens - 1)) : row_base + n - 1;
+        if (VOXZIP_IN_RANGE(p.status, drow >= 0 && drow < p.rows)) {
+            *reinterpret_cast<uint4 *>(p.k_cache + drow * D + lane * 8) = kn4;
+            *reinterpret_cast<uint4 *>(p.v_cache + drow * D + lane * 8) = vn4;
+        }
         if (lane == 0) p.pos[row_base + n - 1] = p.new_pos[ui.b];
     }
     if (tid == 0) {
@@ -273,6 +275,8 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                 const bool is_k = i < ntiles;
                 const int tile = is_k ? i : i - ntiles;
                 const int32_t y = kPaged ? tile_rows[tile] : (int32_t)(row_base + j0 + tile * kTile);
+                // (a TMA load outside the map reads zeros, so a bad row is only recorded)
+                (void)VOXZIP_IN_RANGE(p.status, y >= 0 && (int64_t)y < p.rows);
                 uint8_t *dst = stages + s * Lay::kStageBytes;
 #pragma unroll
                 for (int h = 0; h < kHalves; ++h)
@@ -287,7 +291,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                         const int at = ak ? ia : ia - ntiles;
                         const int rows = min(kTile, cnt - at * kTile);
                         const int64_t row0 = kPaged ? (int64_t)tile_rows[at] : row_base + j0 + (int64_t)at * kTile;
-                        if (rows > 0)
+                        if (rows > 0 && VOXZIP_IN_RANGE(p.status, row0 >= 0 && row0 + rows <= p.rows))
                             ptx::prefetch_l2((ak ? p.k_cache : p.v_cache) + row0 * D, (uint32_t)rows * D * 2);
                     }
                 }
@@ -448,7 +452,8 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                     if (!clustered) {  // Eq. 6: A = gamma * [A, 0] + sum over the heads (a token's four lanes)
                         add += __shfl_xor_sync(0xffffffffu, add, 1);
                         add += __shfl_xor_sync(0xffffffffu, add, 2);
-                        if (valid && qd == 0) sc[lt] = lt == jn ? add : p.gamma * s_old[lt] + add;
+                        if (valid && qd == 0 && VOXZIP_IN_RANGE(p.status, j0 + lt < p.C))
+                            sc[lt] = lt == jn ? add : p.gamma * s_old[lt] + add;
                     }
                 }
                 // Rows past the range may hold anything; zero them so 0 * garbage cannot be NaN.
@@ -570,7 +575,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                 const float4 v = pr[h4];
                 add += v.x * fs[h4 * 4] + v.y * fs[h4 * 4 + 1] + v.z * fs[h4 * 4 + 2] + v.w * fs[h4 * 4 + 3];
             }
-            sc[i] = i == jn ? add : p.gamma * s_old[i] + add;
+            if (VOXZIP_IN_RANGE(p.status, j0 + i < p.C)) sc[i] = i == jn ? add : p.gamma * s_old[i] + add;
         }
     }
     // Sum the CTAs' partial outputs, normalised; CTA r writes slice r of the G x D outputs.
@@ -837,6 +842,7 @@ cudaError_t launch_impl(const voxzip_cache_desc &d, void *k_base, void *v_base, 
     prm.status = status;
     prm.B = d.batch; prm.L = d.layers; prm.Hq = d.q_heads; prm.Hkv = d.kv_heads; prm.G = G;
     prm.C = d.capacity; prm.layer_begin = layer_begin; prm.chunk_cap = chunk_cap; prm.n_hint = nmax;
+    prm.rows = rows;
     prm.gamma = gamma;
     prm.pv = pv;
     const float scale = sm_scale > 0.f ? sm_scale : 1.0f / sqrtf((float)d.head_dim);

@@ -48,6 +48,7 @@ struct EvictParams {
     int32_t budget_stride_b, budget_stride_l, history;
     float recent_frac;
     PageView pv;  // paged instantiations only: K/V rows through the page table, pools as k/v_cache
+    int64_t rows; // K / V rows of the cache, or of the pools
 };
 
 // The unit's budget and its split into T sinks, M recent rows and N history rows.
@@ -188,6 +189,8 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
     uint4 *kc = reinterpret_cast<uint4 *>(static_cast<T *>(p.k_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
     uint4 *vc = reinterpret_cast<uint4 *>(static_cast<T *>(p.v_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
     auto slot_row = [&](int32_t slot) -> int64_t { return kPaged ? paged_row(p.pv, ui.cache_unit, slot) : slot; };
+    auto row_ok = [&](int64_t r) { return !kPaged || (r >= 0 && r < p.rows); };  // checked builds only
+    (void)row_ok;
     const int32_t c_end = n - M;  // history candidates are slots [T, c_end)
 
     // Eq. 9: the N-th best history score, then (only if needed) the position cut among its ties.
@@ -247,7 +250,7 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
                 const int row = sub * kRows + v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
                 if (row < seg) {
                     const int src = src_list[row];
-                    if (src != rank0 + row) {
+                    if (src != rank0 + row && VOXZIP_IN_RANGE(p.status, src >= 0 && src < n && row_ok(slot_row(src)))) {
                         const uint4 *from = (w < kVecPerRow ? kc : vc) + slot_row(src) * kVecPerRow + (w % kVecPerRow);
                         asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
                                          (uint32_t)__cvta_generic_to_shared(&stage[st][v])),
@@ -279,7 +282,7 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
                 const int row = sub * kRows + v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
                 if (row < seg) {
                     const int dst = rank0 + row;
-                    if (src_list[row] != dst) {
+                    if (src_list[row] != dst && VOXZIP_IN_RANGE(p.status, dst < n && row_ok(slot_row(dst)))) {
                         uint4 *to = w < kVecPerRow ? kc : vc;
                         to[slot_row(dst) * kVecPerRow + (w % kVecPerRow)] = stage[st][v];
                     }
@@ -343,6 +346,8 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
     uint4 *kc = reinterpret_cast<uint4 *>(static_cast<T *>(p.k_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
     uint4 *vc = reinterpret_cast<uint4 *>(static_cast<T *>(p.v_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
     auto slot_row = [&](int32_t slot) -> int64_t { return kPaged ? paged_row(p.pv, ui.cache_unit, slot) : slot; };
+    auto row_ok = [&](int64_t r) { return !kPaged || (r >= 0 && r < p.rows); };  // checked builds only
+    (void)row_ok;
 
     // Sinks: the T lowest positions (<= p_lo); recent window: the M highest (>= p_hi). Positions
     // of a unit are unique, so each select cuts exactly.
@@ -448,7 +453,9 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
             const int r = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
             uint4 *base = w < kVecPerRow ? kc : vc;
             const int e = w % kVecPerRow;
-            base[slot_row(holes[r]) * kVecPerRow + e] = base[slot_row(movers[r]) * kVecPerRow + e];
+            if (VOXZIP_IN_RANGE(p.status, holes[r] >= 0 && holes[r] < bud && movers[r] >= bud && movers[r] < n &&
+                                           row_ok(slot_row(holes[r])) && row_ok(slot_row(movers[r]))))
+                base[slot_row(holes[r]) * kVecPerRow + e] = base[slot_row(movers[r]) * kVecPerRow + e];
         }
         for (int r = tid; r < pairs; r += kThreads) {
             sc[holes[r]] = sc[movers[r]];
@@ -521,6 +528,7 @@ cudaError_t launch_evict_policy(const voxzip_cache_desc &d, int32_t layer_begin,
     prm.budget_stride_b = pol.budget_stride_b; prm.budget_stride_l = pol.budget_stride_l;
     prm.history = pol.history;
     prm.pv = PageView{nullptr, nullptr, nullptr, 0};
+    prm.rows = (int64_t)d.batch * d.layers * d.kv_heads * d.capacity;
     const int units = layer_count * d.batch * d.kv_heads;
     const bool bf16 = d.dtype == VOXZIP_BF16, fill = pol.compaction == VOXZIP_COMPACT_FILL;
     if (d.head_dim == 128)
@@ -540,6 +548,7 @@ cudaError_t launch_evict_paged(const voxzip_cache_desc &d, const voxzip_paged_ca
     prm.budget_stride_b = pol.budget_stride_b; prm.budget_stride_l = pol.budget_stride_l;
     prm.history = pol.history;
     prm.pv = PageView{pc.page_table, pc.free_pages, pc.free_count, pc.max_pages};
+    prm.rows = (int64_t)pc.pages * kPageTokens;
     const int units = layer_count * d.batch * d.kv_heads;
     const bool bf16 = d.dtype == VOXZIP_BF16, fill = pol.compaction == VOXZIP_COMPACT_FILL;
     if (d.head_dim == 128)

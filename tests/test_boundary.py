@@ -171,3 +171,8 @@ def test_embed_fuse_is_validated(L, d_model, dtype, keep):
     rc = L.voxzip_embed_fuse(ctypes.byref(e), P, 100, P, P, P, P, 0, None, None, None, None, 0, keep, P, P, P,
                              None, P, 1 << 20, None)
     assert rc == 1
+
+
+@pytest.mark.parametrize("limit", [0, (1 << 20) + 1])
+def test_selftest_limit_is_validated(L, limit):
+    assert L.voxzip_selftest_bounded_wait(limit, None) == 1

@@ -262,3 +262,23 @@ def test_device_errors_set_status_bits_and_skip():
     voxzip_evict(desc, 0, 1, c["k"], c["v"], c["score"], c["pos"], c["len"],
                  torch.tensor([2, 2, 2], dtype=torch.int32, device="cuda"), sink=4)
     assert voxzip_get_status() & DEV_BAD_BUDGET
+
+
+def test_bounded_wait_gives_up_and_reports_timeout():
+    """Failure detection without a GPU fault: a wait nothing can complete gives up after its
+    limit, sets VOXZIP_DEV_TIMEOUT, and the context stays usable (a decode step runs after it)."""
+    from paper_2608_08569_gb300 import DEV_TIMEOUT, voxzip_selftest_bounded_wait
+    voxzip_get_status()
+    voxzip_selftest_bounded_wait(1000)
+    torch.cuda.synchronize()
+    assert voxzip_get_status() == DEV_TIMEOUT
+    desc = CacheDesc(1, 1, 2, 1, 64, 64, torch.bfloat16)
+    c = allocate_cache(desc, "cuda")
+    q = torch.randn(1, 1, 2, 64, device="cuda").to(torch.bfloat16)
+    kv = torch.randn(1, 1, 1, 64, device="cuda").to(torch.bfloat16)
+    out = torch.empty_like(q)
+    voxzip_decode_step(desc, 0, 1, q, kv, kv, torch.zeros(1, dtype=torch.int32, device="cuda"), c["k"], c["v"],
+                       c["score"], c["pos"], c["len"], 0.9, out)
+    torch.cuda.synchronize()
+    assert voxzip_get_status() == 0 and int(c["len"][0, 0, 0]) == 1
+    assert torch.equal(out[0, 0, 0], kv[0, 0, 0]) and torch.equal(out[0, 0, 1], kv[0, 0, 0])
