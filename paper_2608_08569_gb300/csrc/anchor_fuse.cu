@@ -24,7 +24,6 @@
 #include "paged.cuh"
 
 namespace voxzip {
-namespace {
 
 // SMs of the current device (looked up once per device).
 int sm_count() {
@@ -37,6 +36,8 @@ int sm_count() {
     }
     return cached[dev];
 }
+
+namespace {
 
 // acc[e] += element e of a 16-byte vector (4 fp32 or 8 bf16 values, low address first).
 template <typename T>

@@ -5,7 +5,7 @@
 // StreamingLLM baseline).
 //
 // evict_kernel (ordered compaction):
-// One CTA of 256 threads per unit (small enough that every unit of a launch is resident at once):
+// One CTA of 256 threads per unit:
 //   select   MSB-first radix select (4 passes of 8 bits) over an order-preserving 32-bit image of
 //            the history scores gives the N-th best score. Only when that score is tied and not all
 //            tied rows fit does a second select over their positions (ascending) run, so that
@@ -17,7 +17,13 @@
 //            while one is stored. A kept row never moves up (dest = rank <= src). Sources of a
 //            later sub-chunk sit at slots >= its ranks, beyond every destination of an earlier one,
 //            so in-flight loads never see a store; and a barrier after all of a sub-chunk's loads
-//            have landed precedes its stores, so no row is overwritten before it is read.
+//            have landed precedes its stores, so no row is overwritten before it is read. Neither
+//            argument depends on how the rows travel. With many units per launch, every thread
+//            copies 16-byte vectors by cp.async through a narrow ring (8 KB stages, 3 deep, six CTAs
+//            per SM, so every unit is resident at once). A launch of at most two units per SM
+//            leaves too few CTAs for that: each is bound by its own instruction issue and latency,
+//            not by HBM. Its CTAs take a wide ring instead (up to 96 KB of stages, two CTAs per SM)
+//            in which one warp moves each K and V row with one bulk copy in and one bulk copy out.
 //
 // evict_fill_kernel (hole filling): sinks are the T lowest positions and the recent window the M
 // highest (radix selects over the positions), so the cache need not be in time order; the
@@ -35,8 +41,45 @@ namespace {
 
 constexpr int kThreads = 256;
 constexpr int kSegment = 1024;   // ranks listed per compaction segment
-constexpr int kStageVecs = 2;    // 16-byte vectors per thread per sub-chunk (8 KB per CTA)
-constexpr int kPipe = 3;         // sub-chunks in flight
+constexpr uint32_t kEvictWaitLimit = 1u << 22;  // polls before an mbarrier wait gives up
+
+// The narrow compaction ring: every thread copies kVecs 16-byte vectors per sub-chunk by cp.async,
+// kDepth sub-chunks in flight (8 KB stages, six CTAs per SM).
+struct NarrowRing {
+    static constexpr int kVecs = 2, kDepth = 3, kCtasPerSm = 6;
+};
+// The wide ring: one warp moves 32 rows per sub-chunk, each K and V row by one bulk copy in and
+// one out; up to 96 KB of stages (two CTAs per SM).
+template <typename T, int D>
+struct BulkRing {
+    static constexpr int kRows = 32;
+    static constexpr int kRowBytes = D * (int)sizeof(T);
+    static constexpr int kStageBytes = 2 * kRows * kRowBytes;  // K rows, then V rows
+    static constexpr int kDepth = 98304 / kStageBytes < 8 ? 98304 / kStageBytes : 8;
+    static constexpr size_t kBytes = (size_t)kDepth * kStageBytes;
+    static constexpr int kCtasPerSm = 2;
+    static_assert(kDepth >= 3, "a sub-chunk in flight and two stores draining");
+};
+
+// 1-D bulk copies (the async proxy): global -> shared counted on an mbarrier, shared -> global in
+// bulk groups. Addresses 16-byte aligned, sizes multiples of 16.
+__device__ __forceinline__ void bulk_load(void *smem_dst, const void *src, uint32_t bytes, uint64_t *bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                     ptx::smem_u32(smem_dst)),
+                 "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(ptx::smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_store(void *dst, const void *smem_src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(reinterpret_cast<uint64_t>(dst)),
+                 "r"(ptx::smem_u32(smem_src)), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void bulk_wait_read() {  // at most N groups still reading shared memory
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 struct EvictParams {
     void *k_cache, *v_cache;
@@ -156,12 +199,18 @@ __device__ void radix_pass(int shift, int lo, int hi, KeyFn key_of, RadixState &
     st = *shared_st;
 }
 
-template <typename T, int D, bool kPaged>
-__global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p) {
+template <typename T, int D, bool kPaged, bool kWide>
+__global__ void __launch_bounds__(kThreads, kWide ? BulkRing<T, D>::kCtasPerSm : NarrowRing::kCtasPerSm)
+evict_kernel(const EvictParams p) {
     constexpr int kVecPerRow = D * (int)sizeof(T) / 16;  // 16-byte vectors in one K (or V) row
-    constexpr int kRows = kThreads * kStageVecs / (2 * kVecPerRow);
+    using BR = BulkRing<T, D>;
+    constexpr int kStageVecs = NarrowRing::kVecs;
+    constexpr int kPipe = kWide ? BR::kDepth : NarrowRing::kDepth;
+    constexpr int kRows = kWide ? BR::kRows : kThreads * kStageVecs / (2 * kVecPerRow);
     __shared__ int32_t src_list[kSegment];
-    __shared__ uint4 stage[kPipe][kThreads * kStageVecs];
+    __shared__ uint4 ring_static[kWide ? 1 : kPipe][kWide ? 1 : kThreads * kStageVecs];  // narrow ring
+    extern __shared__ uint4 ring_dyn[];                                                  // wide ring
+    __shared__ uint64_t full[kWide ? kPipe : 1];  // wide: the stage's bulk loads have landed
     __shared__ float stage_sc[kPipe][kRows];
     __shared__ int32_t stage_ps[kPipe][kRows];
     __shared__ unsigned hist[256];
@@ -185,6 +234,13 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
     }
     float *sc = p.score + ui.cache_unit * p.C;
     int32_t *ps = p.pos + ui.cache_unit * p.C;
+    if constexpr (kWide) {
+        if (tid == 0) {
+            for (int s = 0; s < kPipe; ++s) ptx::mbar_init(&full[s], 1);
+            ptx::fence_mbar_init();
+        }
+        // (the selection's first barrier orders the initialisation before any use)
+    }
     // K/V rows: the unit's slots (dense), or pool rows through the page table (paged).
     uint4 *kc = reinterpret_cast<uint4 *>(static_cast<T *>(p.k_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
     uint4 *vc = reinterpret_cast<uint4 *>(static_cast<T *>(p.v_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
@@ -219,6 +275,8 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
 
     // Eq. 7-8: ordered, in-place compaction of the kept rows.
     int cursor = 0, rank0 = 0;
+    bool ok = true;          // wide: every mbarrier wait succeeded
+    uint32_t g_sub = 0;      // wide: sub-chunks issued so far (stage and phase of the next one)
     while (cursor < n) {
         int seg = 0;
         while (cursor < n && seg + kThreads <= kSegment) {
@@ -240,8 +298,99 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
         }
         __syncthreads();
 
-        // Move ranks [rank0, rank0 + seg) in sub-chunks of kRows through the cp.async ring.
+        // Move ranks [rank0, rank0 + seg) in sub-chunks of kRows through the ring.
         const int nsub = (seg + kRows - 1) / kRows;
+        if constexpr (kWide) {
+            // One warp: lane l owns row l of every 32-row sub-chunk. Kept rows with consecutive
+            // source slots form runs (split at page boundaries when paged); each run of K (and of V)
+            // comes in by one bulk copy counted on the stage's mbarrier. The rows that move form a
+            // suffix (once an evicted slot precedes a row, one precedes every later row) with
+            // consecutive destinations, so a sub-chunk's moving rows go out by one bulk copy of K
+            // and one of V (two each when they cross a page boundary). Loads run kAhead sub-chunks
+            // ahead of stores, and a stage is reloaded only after the store that read it has read
+            // it. Score and position travel by 4-byte cp.async and plain stores.
+            constexpr int kAhead = kPipe - 2;
+            constexpr uint32_t RB = BR::kRowBytes;
+            if (tid < 32 && ok) {
+                const int lane = tid;
+                for (int it = 0; it < nsub + kAhead; ++it) {
+                    const int sub = it - kAhead;
+                    if (sub >= 0) {
+                        const uint32_t gs = g_sub + (uint32_t)sub;
+                        const int st = (int)(gs % kPipe);
+                        if (!__all_sync(0xffffffffu, ptx::mbar_wait_bounded(&full[st], (gs / kPipe) & 1, kEvictWaitLimit))) {
+                            ok = false;
+                            break;
+                        }
+                        asm volatile("cp.async.wait_group %0;" ::"n"(kAhead - 1) : "memory");
+                        const int row = sub * kRows + lane;
+                        const int dst = rank0 + row;
+                        const bool mv = row < seg && src_list[row] != dst &&
+                                        VOXZIP_IN_RANGE(p.status, dst < n && row_ok(slot_row(dst)));
+                        // The moving rows are a suffix of the sub-chunk with consecutive destinations;
+                        // paged, a page boundary splits them in two.
+                        const bool prev_mv = __shfl_up_sync(0xffffffffu, mv ? 1 : 0, 1) != 0;  // every lane
+                        const bool piece = mv && (lane == 0 || !prev_mv || (kPaged && (dst & (kPageTokens - 1)) == 0));
+                        const unsigned movers = __ballot_sync(0xffffffffu, mv);
+                        const unsigned pieces = __ballot_sync(0xffffffffu, piece);
+                        if (mv) {
+                            sc[dst] = stage_sc[st][lane];
+                            ps[dst] = stage_ps[st][lane];
+                        }
+                        if (piece) {
+                            const unsigned after = lane == 31 ? 0u : (0xffffffffu << (lane + 1));
+                            const unsigned stop = (pieces | ~movers) & after;
+                            const uint32_t bytes = (uint32_t)((stop ? __ffs(stop) - 1 : 32) - lane) * RB;
+                            uint8_t *stage = reinterpret_cast<uint8_t *>(ring_dyn) + st * BR::kStageBytes;
+                            bulk_store(kc + slot_row(dst) * kVecPerRow, stage + lane * RB, bytes);
+                            bulk_store(vc + slot_row(dst) * kVecPerRow, stage + (kRows + lane) * RB, bytes);
+                        }
+                        bulk_commit();
+                    }
+                    if (it < nsub) {
+                        const uint32_t gl = g_sub + (uint32_t)it;
+                        const int st = (int)(gl % kPipe);
+                        bulk_wait_read<kPipe - kAhead>();  // the store that last read this stage is done reading
+                        const int row = it * kRows + lane;
+                        const int src = row < seg ? src_list[row] : -2;
+                        const bool mv = row < seg && src != rank0 + row &&
+                                        VOXZIP_IN_RANGE(p.status, src >= 0 && src < n && row_ok(slot_row(src)));
+                        const int prev_src = __shfl_up_sync(0xffffffffu, src, 1);
+                        const bool prev_mv = __shfl_up_sync(0xffffffffu, mv ? 1 : 0, 1) != 0;
+                        const bool start = mv && (lane == 0 || !prev_mv || src != prev_src + 1 ||
+                                                  (kPaged && (src & (kPageTokens - 1)) == 0));
+                        const unsigned movers = __ballot_sync(0xffffffffu, mv);
+                        const unsigned starts = __ballot_sync(0xffffffffu, start);
+                        if (lane == 0) ptx::mbar_arrive_expect_tx(&full[st], (uint32_t)__popc(movers) * 2u * RB);
+                        __syncwarp();
+                        if (start) {  // this lane's run: up to the next run start or the next row that stays
+                            const unsigned after = lane == 31 ? 0u : (0xffffffffu << (lane + 1));
+                            const unsigned stop = (starts | ~movers) & after;
+                            const int len = (stop ? __ffs(stop) - 1 : 32) - lane;
+                            uint8_t *stage = reinterpret_cast<uint8_t *>(ring_dyn) + st * BR::kStageBytes;
+                            bulk_load(stage + lane * RB, kc + slot_row(src) * kVecPerRow, (uint32_t)len * RB, &full[st]);
+                            bulk_load(stage + (kRows + lane) * RB, vc + slot_row(src) * kVecPerRow, (uint32_t)len * RB,
+                                      &full[st]);
+                        }
+                        if (mv) {
+                            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(ptx::smem_u32(&stage_sc[st][lane])),
+                                         "l"(sc + src)
+                                         : "memory");
+                            asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(ptx::smem_u32(&stage_ps[st][lane])),
+                                         "l"(ps + src)
+                                         : "memory");
+                        }
+                    }
+                    // One 4-byte copy group per iteration (empty in the drain), so that the group of
+                    // the sub-chunk stored next is always the kAhead-th most recent.
+                    asm volatile("cp.async.commit_group;" ::: "memory");
+                }
+                bulk_wait_read<0>();  // the next segment may refill every stage
+                asm volatile("cp.async.wait_all;" ::: "memory");
+            }
+            g_sub += (uint32_t)nsub;
+            __syncthreads();  // src_list is free for the next segment
+        } else {
         auto load_sub = [&](int sub) {
             const int st = sub % kPipe;
 #pragma unroll
@@ -253,7 +402,7 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
                     if (src != rank0 + row && VOXZIP_IN_RANGE(p.status, src >= 0 && src < n && row_ok(slot_row(src)))) {
                         const uint4 *from = (w < kVecPerRow ? kc : vc) + slot_row(src) * kVecPerRow + (w % kVecPerRow);
                         asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(
-                                         (uint32_t)__cvta_generic_to_shared(&stage[st][v])),
+                                         (uint32_t)__cvta_generic_to_shared(&ring_static[st][v])),
                                      "l"(from)
                                      : "memory");
                     }
@@ -284,7 +433,7 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
                     const int dst = rank0 + row;
                     if (src_list[row] != dst && VOXZIP_IN_RANGE(p.status, dst < n && row_ok(slot_row(dst)))) {
                         uint4 *to = w < kVecPerRow ? kc : vc;
-                        to[slot_row(dst) * kVecPerRow + (w % kVecPerRow)] = stage[st][v];
+                        to[slot_row(dst) * kVecPerRow + (w % kVecPerRow)] = ring_static[st][v];
                     }
                 }
             }
@@ -308,7 +457,18 @@ __global__ void __launch_bounds__(kThreads, 6) evict_kernel(const EvictParams p)
                 __syncthreads();  // its stage is drained before the next refill
             }
         }
+        }
         rank0 += seg;
+    }
+    if constexpr (kWide) {
+        if (tid < 32) {
+            if (!ok) {  // a wait gave up: let the loads still in flight land (bounded) before leaving
+                raise_status(p.status, VOXZIP_DEV_TIMEOUT);
+                for (uint32_t g = g_sub > (uint32_t)kPipe ? g_sub - kPipe : 0u; g < g_sub; ++g)
+                    (void)ptx::mbar_wait_bounded(&full[g % kPipe], (g / kPipe) & 1, kEvictWaitLimit);
+            }
+            bulk_wait_all();  // this lane's bulk stores are complete
+        }
     }
     if (tid == 0) p.len[ui.cache_unit] = rank0;  // == budget
     if constexpr (kPaged) {  // pages past the one holding slot bud go back to the pool
@@ -480,10 +640,23 @@ template <typename T, int D, bool kPaged = false>
 cudaError_t launch_t(const EvictParams &prm, int units, bool fill, cudaStream_t stream) {
     // A programmatic dependent of the previous kernel (the decode step): the kernels wait for it
     // before their first read, and a launch without that attribute is the fallback.
-    void (*kern)(EvictParams) = fill ? evict_fill_kernel<T, D, kPaged> : evict_kernel<T, D, kPaged>;
+    const bool wide = !fill && units <= BulkRing<T, D>::kCtasPerSm * sm_count();
+    void (*kern)(EvictParams) = fill ? evict_fill_kernel<T, D, kPaged>
+                                     : (wide ? evict_kernel<T, D, kPaged, true> : evict_kernel<T, D, kPaged, false>);
+    if (wide) {  // above the default 48 KB of dynamic shared memory: opt in once
+        static bool configured = false;
+        if (!configured) {
+            const cudaError_t e = cudaFuncSetAttribute(evict_kernel<T, D, kPaged, true>,
+                                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                       (int)BulkRing<T, D>::kBytes);
+            if (e != cudaSuccess) return e;
+            configured = true;
+        }
+    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)units, 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = wide ? BulkRing<T, D>::kBytes : 0;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

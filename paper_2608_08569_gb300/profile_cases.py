@@ -2,10 +2,11 @@
 
     python -m paper_2608_08569_gb300.profile_cases decode [reps]   # decode step, 60-min 20x steady state
     python -m paper_2608_08569_gb300.profile_cases evict [reps]    # one eviction of that state
+    python -m paper_2608_08569_gb300.profile_cases evict_small [reps]  # eviction, 10-min 4x steady state
     python -m paper_2608_08569_gb300.profile_cases fuse [reps]     # stage 1 of the 60-min request, 4 layers
 
 Each case holds at most a few GB on the device (decode / evict: 0.94 GB of K/V, 4 sequences x 48
-layers x 4 kv-heads at about 2 330 tokens), restores the same seeded state before every launch and
+layers x 4 kv-heads at about 2 330 tokens; evict_small: 0.2 GB, one sequence at 2 035), restores the same seeded state before every launch and
 synchronises after it, so `-s <reps-1> -c 1` captures one steady launch. Inputs are seeded synthetic
 tensors; nothing here checks results (the tests do).
 """
@@ -22,9 +23,11 @@ from . import workloads as W
 def run(mode: str, reps: int = 6) -> None:
     g = torch.Generator(device="cuda")
     g.manual_seed(1)
-    if mode in ("decode", "evict"):
-        B, L, Hq, H, D = 4, 48, 32, 4, 128
-        n = 2333 if mode == "evict" else 2330      # 60-min 20x: budget 2 301, up to 32 steps past it
+    if mode in ("decode", "evict", "evict_small"):
+        B, L, Hq, H, D = (1 if mode == "evict_small" else 4), 48, 32, 4, 128
+        # 60-min 20x: budget 2 301, up to 32 steps past it; 10-min 4x: budget 2 003
+        budget = 2003 if mode == "evict_small" else 2301
+        n = budget + 32 if mode != "decode" else 2330
         cap = n + 64
         desc = CacheDesc(B, L, Hq, H, D, cap, torch.bfloat16)
         c = allocate_cache(desc)
@@ -39,7 +42,7 @@ def run(mode: str, reps: int = 6) -> None:
         vn = torch.randn(L, B, H, D, device="cuda", generator=g).to(torch.bfloat16)
         out = torch.empty_like(q)
         npos = torch.full((B,), 99999, dtype=torch.int32, device="cuda")
-        bud = torch.full((B,), 2301, dtype=torch.int32, device="cuda")
+        bud = torch.full((B,), budget, dtype=torch.int32, device="cuda")
         for _ in range(reps):
             for k in c:
                 c[k].copy_(ref[k])
@@ -67,7 +70,7 @@ def run(mode: str, reps: int = 6) -> None:
                                c["pos"], c["len"])
             torch.cuda.synchronize()
     else:
-        raise SystemExit(f"unknown case {mode!r}: decode, evict or fuse")
+        raise SystemExit(f"unknown case {mode!r}: decode, evict, evict_small or fuse")
     if voxzip_get_status() != 0:
         raise SystemExit("device status word set")
     print("ok", mode)
