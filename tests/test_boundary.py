@@ -36,6 +36,16 @@ def test_library_exports_every_declared_symbol(L):
     assert not missing, missing
 
 
+def test_checked_variant_builds_and_exports_every_declared_symbol():
+    """The range-checked build (-DVOXZIP_CHECKED) compiles its guarded accesses, which the regular
+    build leaves out, and exports the same C ABI."""
+    path = B.build_library(checked=True)
+    assert path == B.CHECKED_LIB_PATH and path != B.LIB_PATH
+    lib = ctypes.CDLL(path)
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
 def test_library_is_sm103a_shared_object(L):
     assert os.path.dirname(B.LIB_PATH) == os.path.dirname(os.path.abspath(B.__file__))
     assert L.voxzip_version() == 100
