@@ -239,7 +239,8 @@ evict_kernel(const EvictParams p) {
             for (int s = 0; s < kPipe; ++s) ptx::mbar_init(&full[s], 1);
             ptx::fence_mbar_init();
         }
-        // (the selection's first barrier orders the initialisation before any use)
+        // (the next block-wide barrier, in the selection or else in the compaction's first scan,
+        // orders the initialisation before any use)
     }
     // K/V rows: the unit's slots (dense), or pool rows through the page table (paged).
     uint4 *kc = reinterpret_cast<uint4 *>(static_cast<T *>(p.k_cache) + (kPaged ? 0 : ui.cache_unit * p.C * D));
