@@ -277,7 +277,9 @@ evict_kernel(const EvictParams p) {
     // Eq. 7-8: ordered, in-place compaction of the kept rows.
     int cursor = 0, rank0 = 0;
     bool ok = true;          // wide: every mbarrier wait succeeded
-    uint32_t g_sub = 0;      // wide: sub-chunks issued so far (stage and phase of the next one)
+    uint32_t g_sub = 0;      // wide: sub-chunks of earlier segments (stage and phase of the next one)
+    uint32_t g_loaded = 0;   // wide: sub-chunks whose loads were issued
+    uint32_t g_stored = 0;   // wide: sub-chunks whose loads were seen to land
     while (cursor < n) {
         int seg = 0;
         while (cursor < n && seg + kThreads <= kSegment) {
@@ -323,6 +325,7 @@ evict_kernel(const EvictParams p) {
                             ok = false;
                             break;
                         }
+                        g_stored = gs + 1;
                         asm volatile("cp.async.wait_group %0;" ::"n"(kAhead - 1) : "memory");
                         const int row = sub * kRows + lane;
                         const int dst = rank0 + row;
@@ -381,6 +384,7 @@ evict_kernel(const EvictParams p) {
                                          "l"(ps + src)
                                          : "memory");
                         }
+                        g_loaded = gl + 1;
                     }
                     // One 4-byte copy group per iteration (empty in the drain), so that the group of
                     // the sub-chunk stored next is always the kAhead-th most recent.
@@ -465,8 +469,9 @@ evict_kernel(const EvictParams p) {
         if (tid < 32) {
             if (!ok) {  // a wait gave up: let the loads still in flight land (bounded) before leaving
                 raise_status(p.status, VOXZIP_DEV_TIMEOUT);
-                for (uint32_t g = g_sub > (uint32_t)kPipe ? g_sub - kPipe : 0u; g < g_sub; ++g)
+                for (uint32_t g = g_stored; g < g_loaded; ++g)
                     (void)ptx::mbar_wait_bounded(&full[g % kPipe], (g / kPipe) & 1, kEvictWaitLimit);
+                asm volatile("cp.async.wait_all;" ::: "memory");
             }
             bulk_wait_all();  // this lane's bulk stores are complete
         }
