@@ -18,12 +18,14 @@
 //            later sub-chunk sit at slots >= its ranks, beyond every destination of an earlier one,
 //            so in-flight loads never see a store; and a barrier after all of a sub-chunk's loads
 //            have landed precedes its stores, so no row is overwritten before it is read. Neither
-//            argument depends on how the rows travel. With many units per launch, every thread
-//            copies 16-byte vectors by cp.async through a narrow ring (8 KB stages, 3 deep, six CTAs
-//            per SM, so every unit is resident at once). A launch of at most two units per SM
-//            leaves too few CTAs for that: each is bound by its own instruction issue and latency,
-//            not by HBM. Its CTAs take a wide ring instead (up to 96 KB of stages, two CTAs per SM)
-//            in which one warp moves each K and V row with one bulk copy in and one bulk copy out.
+//            argument depends on how the rows travel:
+//            - many units per launch: every thread copies 16-byte vectors by cp.async through a
+//              narrow ring (8 KB stages, 3 deep, six CTAs per SM, so a 48-layer launch of four
+//              sequences is resident at once);
+//            - at most two units per SM: that few CTAs would each be bound by their own instruction
+//              issue and latency, not by HBM. They take a wide ring instead (up to 96 KB of stages,
+//              two CTAs per SM), in which one warp moves each run of consecutive source rows in,
+//              and each sub-chunk's moving rows out, by 1-D bulk copies.
 //
 // evict_fill_kernel (hole filling): sinks are the T lowest positions and the recent window the M
 // highest (radix selects over the positions), so the cache need not be in time order; the
