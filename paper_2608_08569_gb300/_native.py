@@ -263,6 +263,8 @@ def voxzip_anchor_fuse_paged(desc: CacheDesc, pc, k_prefill, v_prefill, in_len, 
         _need(t, name, torch.int32, (B,))
     _need(span_off, "span_off", torch.int32, (B + 1,))
     num_spans = span_start.numel()
+    for name, t in (("span_start", span_start), ("span_end", span_end), ("span_groups", span_groups)):
+        _need(t, name, torch.int32, (num_spans,))
     _check_dense_state(desc, pc["score"], pc["pos"], pc["len"])
     if slot_map is not None:
         _need(slot_map, "slot_map", torch.int32, (B, stride))
@@ -275,6 +277,7 @@ def voxzip_anchor_fuse_paged(desc: CacheDesc, pc, k_prefill, v_prefill, in_len, 
     need = int(lib().voxzip_anchor_fuse_paged_workspace_size(ctypes.byref(d), int(stride), int(num_spans)))
     if workspace is None or workspace.numel() < need:
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=k_prefill.device)
+    _need(workspace, "workspace", torch.uint8)
     _check("voxzip_anchor_fuse_paged", lib().voxzip_anchor_fuse_paged(
         ctypes.byref(d), ctypes.byref(ps), _ptr(k_prefill), _ptr(v_prefill), int(stride), _ptr(in_len),
         _ptr(audio_begin), _ptr(audio_len), _ptr(span_off), int(num_spans), _ptr(span_start), _ptr(span_end),
