@@ -77,6 +77,26 @@ def pin_stage1_hand(orc):
     np.testing.assert_allclose(r["exact"], _rows(m["expected_rows_with_anchor"]), rtol=0, atol=1e-12)
 
 
+def pin_run_unit_fuses_k_and_v_with_their_own_anchors(orc):
+    """A whole unit (stage 1, then one decode step, no eviction) fuses K with the K anchors and V
+    with the V anchors. With V's rows twice K's (the hand-worked stage-1 example) and V's anchors the
+    negated K anchors, the example's means M and anchored means A give, row by row, K = A and
+    V = 2M - (A - M) = 3M - A (Eq. 4 and the anchor addition are linear in the rows)."""
+    g = _golden("stage1_hand.json")
+    x = np.array([[t, t * t] for t in range(g["in_len"])], float)
+    anchor = np.array([[100.0 * (k + 1), -(k + 1.0)] for k in range(sum(g["span_groups"]))])
+    M, A = _rows(g["expected_rows"]), _rows(g["expected_rows_with_anchor"])
+    n1, D = len(M), 2
+    cap = n1 + 4
+    r = orc.run_unit(x, 2.0 * x, g["in_len"], g["audio_begin"], g["audio_len"], g["span_start"], g["span_end"],
+                     g["span_groups"], q=np.zeros((1, 1, D)), k_new=np.zeros((1, D)), v_new=np.zeros((1, D)),
+                     new_pos=[1000], gamma=0.9, scale=1.0, interval=1000, budget=cap, capacity=cap,
+                     anchor_k=anchor, anchor_v=-anchor)
+    assert r["stage1_len"] == n1 and r["n"] == n1 + 1
+    np.testing.assert_allclose(r["K"][:n1], A, rtol=1e-6, atol=1e-6)
+    np.testing.assert_allclose(r["V"][:n1], 3.0 * M - A, rtol=1e-6, atol=1e-5)
+
+
 def pin_stage1_bf16_rounding(orc):
     """Hand-worked round-to-nearest-even of fp32 group means into a bf16 cache."""
     for c in _golden("stage1_bf16_rounding.json")["cases"]:

@@ -75,6 +75,15 @@ MUTATIONS = [
      "(int32_t)floor((double)recent_frac * (double)budget)"),
     ("margin against the wrong runner-up", "*margin = c[N - 1].score - c[N].score;",
      "*margin = c[N - 1].score - c[N + 1 < nc ? N + 1 : N].score;"),
+    ("ordered compaction leaves K behind",
+     "                memmove(K + (int64_t)w * D, K + (int64_t)j * D, sizeof(double) * (size_t)D);\n", ""),
+    ("ordered compaction leaves V behind",
+     "                memmove(V + (int64_t)w * D, V + (int64_t)j * D, sizeof(double) * (size_t)D);\n", ""),
+    ("hole filling leaves V behind",
+     "            memcpy(V + (int64_t)h * D, V + (int64_t)j * D, sizeof(double) * (size_t)D);\n", ""),
+    ("V fused with the K anchors",
+     "span_groups, D, xv, anchor_v, cache_is_bf16,", "span_groups, D, xv, anchor_k, cache_is_bf16,"),
+    ("score sums one head of the group", "            score[j] += p;", "            score[j] += h == 0 ? p : 0.0;"),
 ]
 
 
