@@ -84,6 +84,17 @@ MUTATIONS = [
     ("V fused with the K anchors",
      "span_groups, D, xv, anchor_v, cache_is_bf16,", "span_groups, D, xv, anchor_k, cache_is_bf16,"),
     ("score sums one head of the group", "            score[j] += p;", "            score[j] += h == 0 ? p : 0.0;"),
+    ("append writes k_new into V", "        V[(int64_t)n * D + d] = v_new[d];", "        V[(int64_t)n * D + d] = k_new[d];"),
+    ("history candidates overlap the recent window", "    const int32_t nc = n - M - T;",
+     "    const int32_t nc = n - T;"),
+    ("ties broken by slot instead of position",
+     "        return 1;\n    return (x->pos > y->pos) - (x->pos < y->pos);\n}\n\nstatic int position_order",
+     "        return 1;\n    return (x->slot > y->slot) - (x->slot < y->slot);\n}\n\nstatic int position_order"),
+    ("Eq. 3 multiplies before dividing", "double fs = floor((double)La * (t_start[i] / tau_total));",
+     "double fs = floor((double)La * t_start[i] / tau_total);"),
+    ("eviction one step late", "        if (t % interval == 0) {", "        if (t > 1 && (t - 1) % interval == 0) {"),
+    ("hole filling orders by slot on a scrambled cache", "position_order);\n    for (int32_t r = 0; r < T; ++r)",
+     "candidate_order);\n    for (int32_t r = 0; r < T; ++r)"),
 ]
 
 
