@@ -27,6 +27,11 @@ def test_golden_fixture():
     np.testing.assert_array_equal(r["end"], g["expected_end"])
     np.testing.assert_array_equal(r["groups"], g["expected_groups"])
     np.testing.assert_array_equal(r["seg_index"], g["expected_seg_index"])
+    e = g["boundary"]  # a segment on exact token boundaries (the order of Eq. 3's operations shows)
+    r = voxzip_segments_to_spans(e["t_start"], e["t_end"], e["confidence"], e["text_len"], e["tau_total"], e["La"],
+                                 e["audio_begin"], e["threshold"])
+    np.testing.assert_array_equal(r["start"], e["expected_start"])
+    np.testing.assert_array_equal(r["end"], e["expected_end"])
 
 
 @pytest.mark.parametrize("name", sorted(W.EMBED_CONFIGS))
