@@ -249,6 +249,11 @@ def pin_segments_hand(orc):
                               e["La"], e["audio_begin"], e["threshold"])
     np.testing.assert_array_equal(r["start"], e["expected_start"])
     np.testing.assert_array_equal(r["end"], e["expected_end"])
+    e = g["nested"]  # a segment inside the previous one: clipped to an empty span that keeps its text rows
+    r = orc.segments_to_spans(e["t_start"], e["t_end"], e["confidence"], e["text_len"], e["tau_total"],
+                              e["La"], e["audio_begin"], e["threshold"])
+    for k in ("start", "end", "groups", "seg_index"):
+        np.testing.assert_array_equal(r[k], e["expected_" + k], err_msg=k)
 
 
 def pin_segments_properties(orc):

@@ -93,6 +93,15 @@ MUTATIONS = [
     ("Eq. 3 multiplies before dividing", "double fs = floor((double)La * (t_start[i] / tau_total));",
      "double fs = floor((double)La * t_start[i] / tau_total);"),
     ("eviction one step late", "        if (t % interval == 0) {", "        if (t > 1 && (t - 1) % interval == 0) {"),
+    ("segments emptied by clipping are dropped", "        span_start[kept] = (int32_t)(audio_begin + s);",
+     "        if (e == s)\n            continue;\n        span_start[kept] = (int32_t)(audio_begin + s);"),
+    ("clipped end not raised to the start", "        if (e < s)\n            e = s;\n", ""),
+    ("clamp at L_a - 1", "int64_t e = fe < 0.0 ? 0 : (fe > (double)La ? La : (int64_t)fe);",
+     "int64_t e = fe < 0.0 ? 0 : (fe > (double)La - 1 ? La - 1 : (int64_t)fe);"),
+    ("no eviction one row over the budget", "    if (n <= budget)\n        return VZO_OK;",
+     "    if (n <= budget + 1)\n        return VZO_OK;"),
+    ("stage-1 scores not reset", "    for (int32_t j = 0; j < n; ++j)\n        score[j] = 0.0;\n\n    int32_t ev = 0;",
+     "    for (int32_t j = 0; j < n; ++j)\n        score[j] = 1.0;\n\n    int32_t ev = 0;"),
     ("hole filling orders by slot on a scrambled cache", "position_order);\n    for (int32_t r = 0; r < T; ++r)",
      "candidate_order);\n    for (int32_t r = 0; r < T; ++r)"),
 ]

@@ -32,6 +32,11 @@ def test_golden_fixture():
                                  e["audio_begin"], e["threshold"])
     np.testing.assert_array_equal(r["start"], e["expected_start"])
     np.testing.assert_array_equal(r["end"], e["expected_end"])
+    e = g["nested"]  # a segment inside the previous one: an empty span that keeps its text rows
+    r = voxzip_segments_to_spans(e["t_start"], e["t_end"], e["confidence"], e["text_len"], e["tau_total"], e["La"],
+                                 e["audio_begin"], e["threshold"])
+    for k in ("start", "end", "groups", "seg_index"):
+        np.testing.assert_array_equal(r[k], e["expected_" + k], err_msg=k)
 
 
 @pytest.mark.parametrize("name", sorted(W.EMBED_CONFIGS))
