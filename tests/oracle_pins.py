@@ -97,6 +97,18 @@ def pin_run_unit_fuses_k_and_v_with_their_own_anchors(orc):
     np.testing.assert_allclose(r["V"][:n1], 3.0 * M - A, rtol=1e-6, atol=1e-5)
 
 
+def pin_stage1_fp32_accumulation(orc):
+    """Hand-worked IEEE cases for the stored group mean: an fp32 sum in token order (not the exact
+    mean rounded once), and the anchor added in fp32 before the one rounding to bf16."""
+    for c in _golden("stage1_fp32_accumulation.json")["cases"]:
+        rows = np.array(c["rows"], float)[:, None].repeat(2, axis=1)
+        n = len(rows)
+        anchor = None if c["anchor"] is None else np.full((1, 2), float(c["anchor"]))
+        r = orc.stage1(rows, n, 0, n, [0], [n], [1], anchor=anchor, cache_is_bf16=c["cache"] == "bf16")
+        assert r["n"] == 1
+        assert r["stored"][0, 0] == c["stored"], (c, r["stored"][0, 0])
+
+
 def pin_stage1_bf16_rounding(orc):
     """Hand-worked round-to-nearest-even of fp32 group means into a bf16 cache."""
     for c in _golden("stage1_bf16_rounding.json")["cases"]:

@@ -102,6 +102,11 @@ MUTATIONS = [
      "    if (n <= budget + 1)\n        return VZO_OK;"),
     ("stage-1 scores not reset", "    for (int32_t j = 0; j < n; ++j)\n        score[j] = 0.0;\n\n    int32_t ev = 0;",
      "    for (int32_t j = 0; j < n; ++j)\n        score[j] = 1.0;\n\n    int32_t ev = 0;"),
+    ("stored mean taken from the fp64 sum", "float stored = acc / (float)(hi - lo);",
+     "float stored = (float)(sum / (double)(hi - lo));"),
+    ("anchor added after the cache rounding",
+     "out_stored[(int64_t)slot * D + d] = cache_is_bf16 ? bf16_round(stored) : (double)stored;",
+     "out_stored[(int64_t)slot * D + d] = cache_is_bf16 ? bf16_round(acc / (float)(hi - lo)) + (anchor ? (float)anchor[(anchor_row + j) * D + d] : 0.0f) : (double)stored;"),
     ("hole filling orders by slot on a scrambled cache", "position_order);\n    for (int32_t r = 0; r < T; ++r)",
      "candidate_order);\n    for (int32_t r = 0; r < T; ++r)"),
 ]
