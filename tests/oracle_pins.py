@@ -386,6 +386,16 @@ def pin_decode_full_attention(orc):
         cum[:len(Kall)] += w.sum(0).numpy()
         np.testing.assert_allclose(c.score[:c.n], cum[:c.n], rtol=1e-12, atol=1e-14)
     np.testing.assert_array_equal(c.pos[n0:c.n], 1000 + np.arange(steps))
+    # A caller-chosen softmax scale (the C ABI's sm_scale) replaces 1/sqrt(D): SDPA with that scale.
+    c = _random_cache(rng, n0, D, n0 + 1)
+    q = rng.standard_normal((G, D))
+    kn, vn = rng.standard_normal(D), rng.standard_normal(D)
+    out = orc.decode_step(c, q, kn, vn, 2000, 1.0, 0.3)
+    kt = torch.from_numpy(c.K[:c.n].copy())[None, None].expand(1, G, -1, -1)
+    vt = torch.from_numpy(c.V[:c.n].copy())[None, None].expand(1, G, -1, -1)
+    ref = torch.nn.functional.scaled_dot_product_attention(torch.from_numpy(q)[None, :, None, :], kt, vt,
+                                                           scale=0.3)[0, :, 0].numpy()
+    np.testing.assert_allclose(out, ref, rtol=1e-10, atol=1e-12)
 
 
 def pin_decode_total_mass(orc):

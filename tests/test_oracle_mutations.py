@@ -107,6 +107,11 @@ MUTATIONS = [
     ("anchor added after the cache rounding",
      "out_stored[(int64_t)slot * D + d] = cache_is_bf16 ? bf16_round(stored) : (double)stored;",
      "out_stored[(int64_t)slot * D + d] = cache_is_bf16 ? bf16_round(acc / (float)(hi - lo)) + (anchor ? (float)anchor[(anchor_row + j) * D + d] : 0.0f) : (double)stored;"),
+    ("custom softmax scale ignored", "logit[j] = dot * scale;", "logit[j] = dot / sqrt((double)D);"),
+    ("top-N candidates include the sinks", "    const int32_t nc = n - M - T;\n    vzo_candidate *c = all + T;",
+     "    const int32_t nc = n - M;\n    vzo_candidate *c = all;"),
+    ("append overwrites the last row", "        K[(int64_t)n * D + d] = k_new[d];\n        V[(int64_t)n * D + d] = v_new[d];",
+     "        K[(int64_t)(n > 0 ? n - 1 : 0) * D + d] = k_new[d];\n        V[(int64_t)(n > 0 ? n - 1 : 0) * D + d] = v_new[d];"),
     ("hole filling orders by slot on a scrambled cache", "position_order);\n    for (int32_t r = 0; r < T; ++r)",
      "candidate_order);\n    for (int32_t r = 0; r < T; ++r)"),
 ]
