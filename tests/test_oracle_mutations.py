@@ -112,6 +112,10 @@ MUTATIONS = [
      "    const int32_t nc = n - M;\n    vzo_candidate *c = all;"),
     ("append overwrites the last row", "        K[(int64_t)n * D + d] = k_new[d];\n        V[(int64_t)n * D + d] = v_new[d];",
      "        K[(int64_t)(n > 0 ? n - 1 : 0) * D + d] = k_new[d];\n        V[(int64_t)(n > 0 ? n - 1 : 0) * D + d] = v_new[d];"),
+    ("kept flags all set", "            kept[j] = keep[j];", "            kept[j] = 1;"),
+    ("no-op eviction reports a zero margin", "    *margin = INFINITY;", "    *margin = 0.0;"),
+    ("length before eviction recorded after it", "            len_before[ev] = n;\n            rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,\n                              &margin[ev], NULL);",
+     "            rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,\n                              &margin[ev], NULL);\n            len_before[ev] = n;"),
     ("hole filling orders by slot on a scrambled cache", "position_order);\n    for (int32_t r = 0; r < T; ++r)",
      "candidate_order);\n    for (int32_t r = 0; r < T; ++r)"),
 ]
