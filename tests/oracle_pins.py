@@ -677,34 +677,37 @@ def pin_run_unit_identity(orc):
 
 
 def pin_run_unit_composition(orc):
-    """run_unit equals stage1 + decode_step + evict called one by one, in the paper's order."""
-    rng = np.random.default_rng(10)
-    D, G, in_len, steps, interval, budget, cap = 8, 2, 50, 10, 4, 14, 60
-    xk = _bf16(rng.standard_normal((in_len, D)))
-    xv = _bf16(rng.standard_normal((in_len, D)))
-    ss, se, sg = _random_spans(rng, 5, 40)
-    q = rng.standard_normal((steps, G, D))
-    kn, vn = _bf16(rng.standard_normal((steps, D))), _bf16(rng.standard_normal((steps, D)))
-    npos = in_len + np.arange(steps)
-    r = orc.run_unit(xk, xv, in_len, 5, 40, ss, se, sg, q=q, k_new=kn, v_new=vn, new_pos=npos,
-                     gamma=0.9, scale=0.3, interval=interval, budget=budget, capacity=cap,
-                     cache_is_bf16=True)
-    sk = orc.stage1(xk, in_len, 5, 40, ss, se, sg, cache_is_bf16=True, capacity=cap)
-    sv = orc.stage1(xv, in_len, 5, 40, ss, se, sg, cache_is_bf16=True, capacity=cap)
-    c = O.UnitCache.from_rows(cap, sk["stored"], sv["stored"], sk["pos"])
-    ev = 0
-    for t in range(1, steps + 1):
-        out = orc.decode_step(c, q[t - 1], kn[t - 1], vn[t - 1], npos[t - 1], 0.9, 0.3)
-        np.testing.assert_array_equal(out, r["out"][t - 1])
-        if t % interval == 0:
-            assert r["len_before"][ev] == c.n
-            margin, _ = orc.evict(c, budget)
-            assert margin == r["margin"][ev]
-            np.testing.assert_array_equal(r["kept_pos"][ev][:c.n], c.pos[:c.n])
-            ev += 1
-    assert r["n"] == c.n
-    np.testing.assert_array_equal(r["K"], c.K[:c.n])
-    np.testing.assert_array_equal(r["score"], c.score[:c.n])
+    """run_unit equals stage1 + decode_step + evict called one by one, in the paper's order, under
+    every eviction policy (with or without history, ordered or hole-filling compaction)."""
+    for history, fill in ((True, False), (False, False), (True, True), (False, True)):
+        rng = np.random.default_rng(10)
+        D, G, in_len, steps, interval, budget, cap = 8, 2, 50, 10, 4, 14, 60
+        xk = _bf16(rng.standard_normal((in_len, D)))
+        xv = _bf16(rng.standard_normal((in_len, D)))
+        ss, se, sg = _random_spans(rng, 5, 40)
+        q = rng.standard_normal((steps, G, D))
+        kn, vn = _bf16(rng.standard_normal((steps, D))), _bf16(rng.standard_normal((steps, D)))
+        npos = in_len + np.arange(steps)
+        r = orc.run_unit(xk, xv, in_len, 5, 40, ss, se, sg, q=q, k_new=kn, v_new=vn, new_pos=npos,
+                         gamma=0.9, scale=0.3, interval=interval, budget=budget, capacity=cap,
+                         cache_is_bf16=True, history=history, fill=fill)
+        sk = orc.stage1(xk, in_len, 5, 40, ss, se, sg, cache_is_bf16=True, capacity=cap)
+        sv = orc.stage1(xv, in_len, 5, 40, ss, se, sg, cache_is_bf16=True, capacity=cap)
+        c = O.UnitCache.from_rows(cap, sk["stored"], sv["stored"], sk["pos"])
+        ev = 0
+        for t in range(1, steps + 1):
+            out = orc.decode_step(c, q[t - 1], kn[t - 1], vn[t - 1], npos[t - 1], 0.9, 0.3)
+            np.testing.assert_array_equal(out, r["out"][t - 1])
+            if t % interval == 0:
+                assert r["len_before"][ev] == c.n
+                margin, _ = orc.evict(c, budget, history=history, fill=fill)
+                assert margin == r["margin"][ev]
+                np.testing.assert_array_equal(r["kept_pos"][ev][:c.n], c.pos[:c.n])
+                ev += 1
+        assert r["n"] == c.n
+        np.testing.assert_array_equal(r["K"], c.K[:c.n])
+        np.testing.assert_array_equal(r["pos"], c.pos[:c.n])
+        np.testing.assert_array_equal(r["score"], c.score[:c.n])
 
 
 ALL_PINS = [v for k, v in sorted(globals().items()) if k.startswith("pin_") and callable(v)]

@@ -116,6 +116,10 @@ MUTATIONS = [
     ("no-op eviction reports a zero margin", "    *margin = INFINITY;", "    *margin = 0.0;"),
     ("length before eviction recorded after it", "            len_before[ev] = n;\n            rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,\n                              &margin[ev], NULL);",
      "            rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,\n                              &margin[ev], NULL);\n            len_before[ev] = n;"),
+    ("a whole run ignores the fill policy", "rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,",
+     "rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, 0, K, V, score, pos,"),
+    ("a whole run ignores the no-history policy", "rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,",
+     "rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, 1, fill, K, V, score, pos,"),
     ("hole filling orders by slot on a scrambled cache", "position_order);\n    for (int32_t r = 0; r < T; ++r)",
      "candidate_order);\n    for (int32_t r = 0; r < T; ++r)"),
 ]
