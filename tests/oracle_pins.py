@@ -678,8 +678,10 @@ def pin_run_unit_identity(orc):
 
 def pin_run_unit_composition(orc):
     """run_unit equals stage1 + decode_step + evict called one by one, in the paper's order, under
-    every eviction policy (with or without history, ordered or hole-filling compaction)."""
-    for history, fill in ((True, False), (False, False), (True, True), (False, True)):
+    every eviction policy (with or without history, ordered or hole-filling compaction) and with
+    other sink counts and recent fractions than the paper's T = 4 and 20%."""
+    for history, fill, sink, rf in ((True, False, 4, 0.2), (False, False, 4, 0.2), (True, True, 4, 0.2),
+                                    (False, True, 4, 0.2), (True, False, 2, 0.35), (True, True, 3, 0.3)):
         rng = np.random.default_rng(10)
         D, G, in_len, steps, interval, budget, cap = 8, 2, 50, 10, 4, 14, 60
         xk = _bf16(rng.standard_normal((in_len, D)))
@@ -690,7 +692,7 @@ def pin_run_unit_composition(orc):
         npos = in_len + np.arange(steps)
         r = orc.run_unit(xk, xv, in_len, 5, 40, ss, se, sg, q=q, k_new=kn, v_new=vn, new_pos=npos,
                          gamma=0.9, scale=0.3, interval=interval, budget=budget, capacity=cap,
-                         cache_is_bf16=True, history=history, fill=fill)
+                         cache_is_bf16=True, history=history, fill=fill, sink=sink, recent_frac=rf)
         sk = orc.stage1(xk, in_len, 5, 40, ss, se, sg, cache_is_bf16=True, capacity=cap)
         sv = orc.stage1(xv, in_len, 5, 40, ss, se, sg, cache_is_bf16=True, capacity=cap)
         c = O.UnitCache.from_rows(cap, sk["stored"], sv["stored"], sk["pos"])
@@ -700,7 +702,7 @@ def pin_run_unit_composition(orc):
             np.testing.assert_array_equal(out, r["out"][t - 1])
             if t % interval == 0:
                 assert r["len_before"][ev] == c.n
-                margin, _ = orc.evict(c, budget, history=history, fill=fill)
+                margin, _ = orc.evict(c, budget, sink, rf, history=history, fill=fill)
                 assert margin == r["margin"][ev]
                 np.testing.assert_array_equal(r["kept_pos"][ev][:c.n], c.pos[:c.n])
                 ev += 1

@@ -120,6 +120,12 @@ MUTATIONS = [
      "rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, 0, K, V, score, pos,"),
     ("a whole run ignores the no-history policy", "rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,",
      "rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, 1, fill, K, V, score, pos,"),
+    ("a whole run ignores the sink count", "rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,",
+     "rc = vzo_evict_ex(D, &n, budget, 4, recent_frac, history, fill, K, V, score, pos,"),
+    ("a whole run ignores the recent fraction", "rc = vzo_evict_ex(D, &n, budget, sink, recent_frac, history, fill, K, V, score, pos,",
+     "rc = vzo_evict_ex(D, &n, budget, sink, 0.2f, history, fill, K, V, score, pos,"),
+    ("a whole run ignores the cache dtype", "D, xk, anchor_k, cache_is_bf16, capacity, scratch, K, pos, slot_map, &n);",
+     "D, xk, anchor_k, 0, capacity, scratch, K, pos, slot_map, &n);"),
     ("hole filling orders by slot on a scrambled cache", "position_order);\n    for (int32_t r = 0; r < T; ++r)",
      "candidate_order);\n    for (int32_t r = 0; r < T; ++r)"),
 ]
