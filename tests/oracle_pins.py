@@ -679,9 +679,10 @@ def pin_run_unit_identity(orc):
 def pin_run_unit_composition(orc):
     """run_unit equals stage1 + decode_step + evict called one by one, in the paper's order, under
     every eviction policy (with or without history, ordered or hole-filling compaction) and with
-    other sink counts and recent fractions than the paper's T = 4 and 20%."""
-    for history, fill, sink, rf in ((True, False, 4, 0.2), (False, False, 4, 0.2), (True, True, 4, 0.2),
-                                    (False, True, 4, 0.2), (True, False, 2, 0.35), (True, True, 3, 0.3)):
+    other sink counts, recent fractions, decays and softmax scales."""
+    for history, fill, sink, rf, gamma, scale in ((True, False, 4, 0.2, 0.9, 0.3), (False, False, 4, 0.2, 0.9, 0.3),
+                                                  (True, True, 4, 0.2, 0.9, 0.3), (False, True, 4, 0.2, 0.9, 0.3),
+                                                  (True, False, 2, 0.35, 0.97, 0.5), (True, True, 3, 0.3, 0.8, 0.2)):
         rng = np.random.default_rng(10)
         D, G, in_len, steps, interval, budget, cap = 8, 2, 50, 10, 4, 14, 60
         xk = _bf16(rng.standard_normal((in_len, D)))
@@ -691,14 +692,14 @@ def pin_run_unit_composition(orc):
         kn, vn = _bf16(rng.standard_normal((steps, D))), _bf16(rng.standard_normal((steps, D)))
         npos = in_len + np.arange(steps)
         r = orc.run_unit(xk, xv, in_len, 5, 40, ss, se, sg, q=q, k_new=kn, v_new=vn, new_pos=npos,
-                         gamma=0.9, scale=0.3, interval=interval, budget=budget, capacity=cap,
+                         gamma=gamma, scale=scale, interval=interval, budget=budget, capacity=cap,
                          cache_is_bf16=True, history=history, fill=fill, sink=sink, recent_frac=rf)
         sk = orc.stage1(xk, in_len, 5, 40, ss, se, sg, cache_is_bf16=True, capacity=cap)
         sv = orc.stage1(xv, in_len, 5, 40, ss, se, sg, cache_is_bf16=True, capacity=cap)
         c = O.UnitCache.from_rows(cap, sk["stored"], sv["stored"], sk["pos"])
         ev = 0
         for t in range(1, steps + 1):
-            out = orc.decode_step(c, q[t - 1], kn[t - 1], vn[t - 1], npos[t - 1], 0.9, 0.3)
+            out = orc.decode_step(c, q[t - 1], kn[t - 1], vn[t - 1], npos[t - 1], gamma, scale)
             np.testing.assert_array_equal(out, r["out"][t - 1])
             if t % interval == 0:
                 assert r["len_before"][ev] == c.n

@@ -126,6 +126,10 @@ MUTATIONS = [
      "rc = vzo_evict_ex(D, &n, budget, sink, 0.2f, history, fill, K, V, score, pos,"),
     ("a whole run ignores the cache dtype", "D, xk, anchor_k, cache_is_bf16, capacity, scratch, K, pos, slot_map, &n);",
      "D, xk, anchor_k, 0, capacity, scratch, K, pos, slot_map, &n);"),
+    ("a whole run decays with a fixed gamma", "v_new + (int64_t)(t - 1) * D, new_pos[t - 1], gamma, scale,",
+     "v_new + (int64_t)(t - 1) * D, new_pos[t - 1], 0.9, scale,"),
+    ("a whole run scales with a fixed factor", "v_new + (int64_t)(t - 1) * D, new_pos[t - 1], gamma, scale,",
+     "v_new + (int64_t)(t - 1) * D, new_pos[t - 1], gamma, 0.3,"),
     ("hole filling orders by slot on a scrambled cache", "position_order);\n    for (int32_t r = 0; r < T; ++r)",
      "candidate_order);\n    for (int32_t r = 0; r < T; ++r)"),
 ]
