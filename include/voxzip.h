@@ -30,7 +30,10 @@
  *                    score  [B][L][Hkv][C]  fp32    decayed accumulated attention (Eq. 6)
  *                    pos    [B][L][Hkv][C]  int32   original token index of each slot
  *                    len    [B][L][Hkv]     int32   cache length n of each unit
- *     Slots [0, n) of a unit are valid and kept in chronological (ascending position) order.
+ *     Slots [0, n) of a unit are valid. Stage 1, decode appends and the ordered eviction keep them
+ *     in chronological (ascending position) order; the hole-filling eviction
+ *     (VOXZIP_COMPACT_FILL of voxzip_evict_ex) does not: it moves kept rows into evicted slots, so
+ *     a unit's slots are then in no particular order. No call depends on slot order.
  */
 #ifndef VOXZIP_H
 #define VOXZIP_H
@@ -129,8 +132,10 @@ size_t voxzip_anchor_fuse_workspace_size(const voxzip_cache_desc *desc, int32_t 
  *
  * Its scratch is a fixed 4 MiB array compiled into the library, held by every GPU that loads the
  * library until the process exits. A request whose voxzip_anchor_fuse_workspace_size exceeds 4 MiB
- * returns VOXZIP_ESCRATCH and launches nothing. The need is about 8 bytes per prompt token plus
- * 8 per span, so 4 MiB covers for instance 32 sequences of 10 000 tokens or 4 of 80 000.
+ * returns VOXZIP_ESCRATCH and launches nothing. The need is 12 bytes per prompt-token slot
+ * (batch x prefill_stride) plus 12 per span, 8 per sequence and under 2.5 KiB of alignment padding:
+ * 4 MiB covers, for instance, 4 sequences of 60 000 tokens or 32 of 8 000 with one span per five
+ * tokens. voxzip_anchor_fuse_workspace_size gives the exact figure to compare against 4 MiB.
  *   - The first call on a device looks up the array's device address (cudaGetSymbolAddress) with
  *     that device current; make that first call before any stream capture.
  *   - Every call on a device shares the array and it keeps the last call's contents; no part of it
@@ -379,6 +384,18 @@ voxzip_status voxzip_get_status(uint32_t *bits, voxzip_stream_t stream);
  * issued, so nothing can fault. Asynchronous on `stream`; VOXZIP_EINVAL for a limit out of range.
  */
 voxzip_status voxzip_selftest_bounded_wait(uint32_t limit, voxzip_stream_t stream);
+
+/*
+ * Measurement helper, not a step of the method: reads `bytes` of device memory at `p` once with
+ * 16-byte loads spread over the whole GPU, as a plain streaming read, and does nothing with the
+ * data (a checksum that no input produces in practice is the only store, to `sink`, a caller-owned
+ * device word). It is the most a single launch of that size can reach, so it serves as the ceiling
+ * a kernel moving the same bytes is measured against. Like the decode and eviction launches it is a
+ * programmatic dependent of the previous kernel on `stream`, so a captured loop of them overlaps
+ * each launch's start with the previous one's tail exactly as a loop of decode steps does.
+ * `p` 16-byte aligned, `bytes` a multiple of 16; VOXZIP_EINVAL otherwise. Asynchronous.
+ */
+voxzip_status voxzip_stream_read(const void *p, size_t bytes, uint32_t *sink, voxzip_stream_t stream);
 
 /* Human-readable name of a status code (static storage). */
 const char *voxzip_status_string(voxzip_status status);

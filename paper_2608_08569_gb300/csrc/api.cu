@@ -2,6 +2,8 @@
 // status word, and dispatch to the kernel launchers. Nothing here allocates device memory. Every
 // entry point opens an NVTX range of its own name (a no-op unless a profiler listens).
 #include <math.h>
+
+#include <atomic>
 #include <nvtx3/nvToolsExt.h>
 
 #include "common.cuh"
@@ -16,18 +18,23 @@ namespace {
 __device__ int32_t g_status_word;
 
 constexpr int kMaxDevices = 64;
-int32_t *g_status_addr[kMaxDevices];  // device address of g_status_word, per device
+// Device address of g_status_word, per device. Host threads may make their first call on a device
+// at the same time: each looks the address up and stores the same value, so atomics make that race
+// well defined without a lock.
+std::atomic<int32_t *> g_status_addr[kMaxDevices];
 
 // Address of the status word on the current device (looked up once per device).
 voxzip_status status_word(int32_t **addr) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return VOXZIP_ECUDA;
-    if (g_status_addr[dev] == nullptr) {
+    int32_t *a = g_status_addr[dev].load(std::memory_order_acquire);
+    if (a == nullptr) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return VOXZIP_ECUDA;
-        g_status_addr[dev] = static_cast<int32_t *>(p);
+        a = static_cast<int32_t *>(p);
+        g_status_addr[dev].store(a, std::memory_order_release);
     }
-    *addr = g_status_addr[dev];
+    *addr = a;
     return VOXZIP_OK;
 }
 

@@ -9,6 +9,8 @@
 // Host code cannot pass the array's name to a kernel (on the host that name is only a stand-in,
 // not a device address), so the device address is looked up once per device with
 // cudaGetSymbolAddress, with that device current, on the first call made on it.
+#include <atomic>
+
 #include "common.cuh"
 
 namespace {
@@ -21,17 +23,19 @@ static __device__ __align__(256) unsigned char g_fuse_scratch[kScratchBytes];
 
 // The status word lives in api.cu; kernels of this file report through the same word.
 constexpr int kMaxDevices = 64;
-void *g_scratch_addr[kMaxDevices];   // device address of g_fuse_scratch, per device
+// Device address of g_fuse_scratch, per device. Two host threads making their first call on one
+// device at once both look it up and store the same value; the atomic makes that well defined.
+std::atomic<void *> g_scratch_addr[kMaxDevices];
 
 voxzip_status scratch_address(void **out) {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return VOXZIP_ECUDA;
-    if (g_scratch_addr[dev] == nullptr) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_fuse_scratch) != cudaSuccess || p == nullptr) return VOXZIP_ECUDA;
-        g_scratch_addr[dev] = p;
+    void *a = g_scratch_addr[dev].load(std::memory_order_acquire);
+    if (a == nullptr) {
+        if (cudaGetSymbolAddress(&a, g_fuse_scratch) != cudaSuccess || a == nullptr) return VOXZIP_ECUDA;
+        g_scratch_addr[dev].store(a, std::memory_order_release);
     }
-    *out = g_scratch_addr[dev];
+    *out = a;
     return VOXZIP_OK;
 }
 

@@ -15,7 +15,7 @@ import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 PARITY_FILES = ["tests/test_gpu_parity.py", "tests/test_gpu_paged.py", "tests/test_gpu_policies.py",
-                "tests/test_gpu_embed.py"]
+                "tests/test_gpu_embed.py", "tests/test_zzzz_no_alloc.py"]
 
 
 @pytest.mark.gpu
