@@ -17,13 +17,13 @@ from ._native import (CacheDesc, EmbedDesc, VoxZipError, allocate_cache, lib, vo
                       voxzip_anchor_fuse_noalloc, voxzip_anchor_fuse_workspace_size, voxzip_decode_step,
                       voxzip_embed_fuse, voxzip_embed_fuse_workspace_size, voxzip_evict, voxzip_evict_ex,
                       voxzip_get_status, voxzip_segments_to_spans)
-from ._native import (voxzip_selftest_bounded_wait,)
+from ._native import (voxzip_selftest_bounded_wait, voxzip_stream_read)
 from ._native import (PAGE_TOKENS, allocate_paged_cache, paged_pages_in_use, voxzip_anchor_fuse_paged,
                       voxzip_decode_step_paged, voxzip_evict_paged, voxzip_paged_init)
 from ._native import (DEV_BAD_BUDGET, DEV_BAD_POSITIONS, DEV_BOUNDS, DEV_BAD_SPANS, DEV_CAPACITY, DEV_LEN_HINT, DEV_TIMEOUT, VOXZIP_ECUDA,
                       VOXZIP_EINVAL, VOXZIP_ESCRATCH, VOXZIP_EUNSUPPORTED, VOXZIP_OK)
 
-__all__ = ["voxzip_selftest_bounded_wait", "PAGE_TOKENS", "allocate_paged_cache", "paged_pages_in_use", "voxzip_anchor_fuse_paged",
+__all__ = ["voxzip_selftest_bounded_wait", "voxzip_stream_read", "PAGE_TOKENS", "allocate_paged_cache", "paged_pages_in_use", "voxzip_anchor_fuse_paged",
            "voxzip_decode_step_paged", "voxzip_evict_paged", "voxzip_paged_init", "CacheDesc", "EmbedDesc", "voxzip_evict_ex", "DEV_BAD_POSITIONS", "DEV_BOUNDS", "voxzip_embed_fuse", "voxzip_embed_fuse_workspace_size",
            "voxzip_segments_to_spans", "VoxZipError", "allocate_cache", "lib", "voxzip_anchor_fuse", "voxzip_anchor_fuse_noalloc",
            "voxzip_anchor_fuse_workspace_size", "voxzip_decode_step", "voxzip_evict", "voxzip_get_status",

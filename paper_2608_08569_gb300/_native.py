@@ -136,6 +136,8 @@ def lib() -> ctypes.CDLL:
                                              _vp]
             L.voxzip_selftest_bounded_wait.argtypes = [ctypes.c_uint32, _vp]
             L.voxzip_selftest_bounded_wait.restype = _i32
+            L.voxzip_stream_read.argtypes = [_vp, _sz, _vp, _vp]
+            L.voxzip_stream_read.restype = _i32
             L.voxzip_segments_to_spans.argtypes = [_i32, _vp, _vp, _vp, _vp, _f64, _i32, _i32, _f64, _vp, _vp, _vp,
                                                    _vp, _vp]
             L.voxzip_embed_fuse.argtypes = [_EP, _vp, _i32, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _i32,
@@ -520,6 +522,15 @@ def voxzip_selftest_bounded_wait(limit: int = 1000, stream=None) -> None:
     """Launches the bounded-wait self-test: a wait that can never complete gives up after `limit`
     polls and sets DEV_TIMEOUT in the status word (read it with voxzip_get_status)."""
     _check("voxzip_selftest_bounded_wait", lib().voxzip_selftest_bounded_wait(int(limit), _stream(stream)))
+
+
+def voxzip_stream_read(buf: torch.Tensor, nbytes: int, sink: torch.Tensor, stream=None) -> None:
+    """Measurement helper: one plain streaming read of the first `nbytes` of `buf` (a multiple of 16),
+    launched like the decode step; `sink` is a one-element int32 device tensor."""
+    if not buf.is_cuda or nbytes > buf.numel() * buf.element_size():
+        raise ValueError("buf must be a device tensor of at least nbytes")
+    _need(sink, "sink", torch.int32)
+    _check("voxzip_stream_read", lib().voxzip_stream_read(_ptr(buf), int(nbytes), _ptr(sink), _stream(stream)))
 
 
 def voxzip_get_status(stream=None) -> int:

@@ -24,6 +24,8 @@
 // row its page-table entry gives, and the CTA that completes a page takes the next one.
 #include <cooperative_groups.h>
 
+#include <type_traits>
+
 #include "common.cuh"
 #include "paged.cuh"
 #include "ptx.cuh"
@@ -88,8 +90,9 @@ struct Layout {
     static constexpr int kStagesOff = 0;                       // the ring; reused for o_w afterwards
     static constexpr int kRingBytes = kStages * kStageBytes;
     static constexpr int kOStride = D + 4;                     // padded row of the output partials
-    static_assert(kRingBytes >= kConsumerWarps * kGP * kOStride * 4, "ring too small to hold the warp partials");
-    static constexpr int kBarOff = kRingBytes;                 // full[kStages], empty[kStages]
+    static constexpr int kOwBytes = kConsumerWarps * kGP * kOStride * 4;
+    static constexpr int kRingAlloc = kRingBytes > kOwBytes ? kRingBytes : (kOwBytes + 1023) / 1024 * 1024;
+    static constexpr int kBarOff = kRingAlloc;                 // full[kStages], empty[kStages]
     static constexpr int kPbufOff = kBarOff + 2 * kStages * 8;
     static constexpr int kPbufBytes = kConsumerWarps * 16 * kGP * 2;
     static constexpr int kStatOff = kPbufOff + kPbufBytes;     // m_w, z_w [warps][kGP]; m_cta, z_cta [kGP]; fac [S][kGP]
@@ -285,7 +288,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                 // now. It costs no shared memory and keeps more of the SM's bytes in flight; its TMA
                 // load then hits L2.
                 if (VOXZIP_DECODE_L2_AHEAD > 0) {
-                    const int ia = i + kStages + VOXZIP_DECODE_L2_AHEAD - 1;
+                    const int ia = i + kStages + VOXZIP_DECODE_L2_AHEAD + (kStages == 2 ? 1 : 0) - 1;
                     if (ia < 2 * ntiles) {
                         const bool ak = ia < ntiles;
                         const int at = ak ? ia : ia - ntiles;
@@ -539,31 +542,71 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     if (!ok) raise_status(p.status, VOXZIP_DEV_TIMEOUT);
     ptx::launch_dependents();  // streaming is over: the next launch may begin its prologue
     __syncthreads();
+    // CTA r writes slice r of the G x D outputs: the CTAs' partial outputs summed, normalised.
+    constexpr int OS = Lay::kOStride;
+    const int o_total = p.G * D;
+    __nv_bfloat16 *og = p.out + (act_row * p.Hq + (int64_t)ui.h * p.G) * D;
     if (clustered) {
         cluster.sync();  // every CTA's m_cta, z_cta, o_cta are final
-        // The unit's per-head maximum m and normaliser Z; fac[r][h] = 2^(m_r - m) / Z.
-        if (tid < GP) {
-            float mr[kMaxCluster], zr[kMaxCluster];
+        // For a cluster of SS CTAs (a power of two), this thread's share of the slice is at most E
+        // elements: all their partials from every CTA are requested before the statistics, so the
+        // reads over the cluster take one round trip.
+        auto combine = [&](auto ss_tag) {
+            constexpr int SS = decltype(ss_tag)::value;
+            constexpr int E = (GP * D / SS + kThreads - 1) / kThreads;
+            const int per = (o_total + SS - 1) / SS;
+            const int lo = rank * per, hi = min(o_total, lo + per);
+            float part[E][SS];
 #pragma unroll
-            for (int r = 0; r < kMaxCluster; ++r) {
-                mr[r] = r < S ? *cluster.map_shared_rank(&m_cta[tid], r) : -INFINITY;
-                zr[r] = r < S ? *cluster.map_shared_rank(&z_cta[tid], r) : 0.f;
+            for (int e = 0; e < E; ++e) {
+                const int i = lo + tid + e * kThreads;
+                const int at = i < hi ? (i / D) * OS + i % D : 0;
+#pragma unroll
+                for (int r = 0; r < SS; ++r) part[e][r] = i < hi ? *cluster.map_shared_rank(&o_cta[at], r) : 0.f;
             }
-            float m = -INFINITY;
+            // The unit's per-head maximum m and normaliser Z; fac[r][h] = 2^(m_r - m) / Z.
+            if (tid < GP) {
+                float mr[SS], zr[SS];
 #pragma unroll
-            for (int r = 0; r < kMaxCluster; ++r) m = fmaxf(m, mr[r]);
-            float z = 0.f;
+                for (int r = 0; r < SS; ++r) {
+                    mr[r] = *cluster.map_shared_rank(&m_cta[tid], r);
+                    zr[r] = *cluster.map_shared_rank(&z_cta[tid], r);
+                }
+                float m = -INFINITY;
 #pragma unroll
-            for (int r = 0; r < kMaxCluster; ++r) {
-                mr[r] = mr[r] == -INFINITY ? 0.f : exp2f(mr[r] - m);
-                z += mr[r] * zr[r];
+                for (int r = 0; r < SS; ++r) m = fmaxf(m, mr[r]);
+                float z = 0.f;
+#pragma unroll
+                for (int r = 0; r < SS; ++r) {
+                    mr[r] = mr[r] == -INFINITY ? 0.f : exp2f(mr[r] - m);
+                    z += mr[r] * zr[r];
+                }
+                const float rzv = tid < p.G ? 1.f / z : 0.f;
+#pragma unroll
+                for (int r = 0; r < SS; ++r) fac[r * GP + tid] = mr[r] * rzv;
             }
-            const float rzv = tid < p.G ? 1.f / z : 0.f;
+            __syncthreads();
 #pragma unroll
-            for (int r = 0; r < kMaxCluster; ++r)
-                if (r < S) fac[r * GP + tid] = mr[r] * rzv;
+            for (int e = 0; e < E; ++e) {
+                const int i = lo + tid + e * kThreads;
+                if (i < hi) {
+                    const int h = i / D;
+                    float o = 0.f;
+#pragma unroll
+                    for (int r = 0; r < SS; ++r) o += fac[r * GP + h] * part[e][r];
+                    og[i] = __float2bfloat16_rn(o);
+                }
+            }
+        };
+        switch (S) {
+            case 2: combine(std::integral_constant<int, 2>{}); break;
+            case 4: combine(std::integral_constant<int, 4>{}); break;
+            case 8: combine(std::integral_constant<int, 8>{}); break;
+            default: combine(std::integral_constant<int, 16>{}); break;
         }
-        __syncthreads();
+        // This CTA is done reading its peers' shared memory; they may leave once all have said so.
+        // The score update below touches only this CTA's own shared memory and global memory.
+        asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
         // Eq. 6 for this CTA's tokens: A = gamma * [A, 0] + sum over the group's heads.
         const float *fs = fac + rank * GP;
         float *sc = p.score + row_base + j0;
@@ -577,31 +620,12 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
             }
             if (VOXZIP_IN_RANGE(p.status, j0 + i < p.C)) sc[i] = i == jn ? add : p.gamma * s_old[i] + add;
         }
-    }
-    // Sum the CTAs' partial outputs, normalised; CTA r writes slice r of the G x D outputs.
-    {
-        const int total = p.G * D, per = (total + S - 1) / S;
-        const int lo = rank * per, hi = min(total, lo + per);
-        __nv_bfloat16 *og = p.out + (act_row * p.Hq + (int64_t)ui.h * p.G) * D;
-        for (int i = lo + tid; i < hi; i += kThreads) {
+    } else {
+        for (int i = tid; i < o_total; i += kThreads) {
             const int h = i / D;
-            const int at = h * Lay::kOStride + i % D;
-            float o;
-            if (clustered) {
-                float part[kMaxCluster];
-#pragma unroll
-                for (int r = 0; r < kMaxCluster; ++r) part[r] = r < S ? *cluster.map_shared_rank(&o_cta[at], r) : 0.f;
-                o = 0.f;
-#pragma unroll
-                for (int r = 0; r < kMaxCluster; ++r)
-                    if (r < S) o += fac[r * GP + h] * part[r];
-            } else {
-                o = o_cta[at] * fac[h];
-            }
-            og[i] = __float2bfloat16_rn(o);
+            og[i] = __float2bfloat16_rn(o_cta[h * OS + i % D] * fac[h]);
         }
     }
-    if (clustered) cluster.sync();  // no CTA leaves while others may still read its shared memory
     if (rank == 0 && tid == 0) {
         p.len[ui.cache_unit] = n;
         if constexpr (kPaged) {  // the next append starts a page: take one now
@@ -611,6 +635,8 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
             }
         }
     }
+    // No CTA leaves while a peer may still read its shared memory.
+    if (clustered) asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 // ---------------------------------------------------------------- host side
@@ -621,11 +647,12 @@ struct Tag {
 
 // Calls f(Tag<D, NT, NS>{}) for the runtime shape; the kernel is instantiated for D in {64, 128},
 // NT in {1, 2} (group <= 8 or <= 16) and a ring of NS in {3, 4, 6, 8} stages.
-constexpr int kRingDepths[] = {3, 4, 6, 8};
+constexpr int kRingDepths[] = {2, 3, 4, 6, 8};
 
 template <int D, int NT, typename F>
 auto dispatch_ns(int NS, F &&f) {
     switch (NS) {
+        case 2: return f(Tag<D, NT, 2>{});
         case 4: return f(Tag<D, NT, 4>{});
         case 6: return f(Tag<D, NT, 6>{});
         case 8: return f(Tag<D, NT, 8>{});

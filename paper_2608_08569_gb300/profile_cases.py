@@ -54,6 +54,19 @@ def run(mode: str, reps: int = 6) -> None:
             else:
                 voxzip_evict(desc, 0, L, c["k"], c["v"], c["score"], c["pos"], c["len"], bud)
             torch.cuda.synchronize()
+        # Algorithmic bytes of one launch, for the summary's traffic ratio. Decode: every K and V row
+        # once, the score read and written, q and out, k_new and v_new and their append, the position.
+        # Eviction: 8 B per slot for the selection, and K, V, score and position read and written for
+        # every kept row that changed slot (counted from the positions before and after).
+        e = 2
+        if mode == "decode":
+            alg = L * B * H * ((n + 1) * (2 * D * e + 8) + (2 * (Hq // H) * D + 4 * D) * e + 4)
+        else:
+            na = c["len"].reshape(-1).long()
+            idx = torch.arange(cap, device="cuda")
+            moved = ((ref["pos"].reshape(-1, cap) != c["pos"].reshape(-1, cap)) & (idx[None] < na[:, None])).sum()
+            alg = 8 * n * L * B * H + 2 * (2 * D * e + 8) * int(moved)
+        print("algorithmic_bytes_per_launch", int(alg))
     elif mode == "fuse":
         w = W.scaled(W.CONFIGS["stress"], layers=4, name="stress_l4")
         sp = W.make_spans(w)
