@@ -54,6 +54,9 @@ def parse_args():
     p.add_argument("--workload", default="stress")
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-targets", action="store_true",
+                   help="skip the decode/evict rooflines at the four target points (60-min and 10-min audio "
+                        "at the 20x and 4x budgets)")
     p.add_argument("--cpu-units", type=int, default=0, help="units in the oracle sample (0: one per core)")
     p.add_argument("--compaction", choices=["ordered", "fill"], default="ordered",
                    help="eviction compaction: ordered (Eq. 7-8, default) or hole filling")
@@ -220,26 +223,34 @@ def evict_bytes(w, n_before, moved_rows):
 # ----------------------------------------------------------------------------- GPU arm
 
 class Runner:
-    def __init__(self, w, device, compaction="ordered", paged=False):
+    """One workload's resident inputs and session. With `share` (a dense Runner of a workload that
+    differs only in its budget), the inputs, the cache memory and the outputs are that runner's."""
+
+    def __init__(self, w, device, compaction="ordered", paged=False, share=None):
         from paper_2608_08569_gb300 import CacheDesc
         from paper_2608_08569_gb300 import workloads as W
         from paper_2608_08569_gb300.session import Session
         self.w = w
         self.dev = device
-        self.spans = W.make_spans(w)
-        i32 = lambda a: torch.as_tensor(np.asarray(a), dtype=torch.int32, device=device)
-        self.span_args = (i32(w.in_len), i32([w.audio_begin] * w.batch), i32(w.audio_len), i32(self.spans.off),
-                          i32(self.spans.start), i32(self.spans.end), i32(self.spans.groups))
-        self.k_pre, self.v_pre = W.make_prefill(w, device)
-        self.q, self.kn, self.vn, self.npos = W.make_steps(w, device)
+        if share is not None:
+            for n in ("spans", "span_args", "k_pre", "v_pre", "q", "kn", "vn", "npos", "out"):
+                setattr(self, n, getattr(share, n))
+        else:
+            self.spans = W.make_spans(w)
+            i32 = lambda a: torch.as_tensor(np.asarray(a), dtype=torch.int32, device=device)
+            self.span_args = (i32(w.in_len), i32([w.audio_begin] * w.batch), i32(w.audio_len), i32(self.spans.off),
+                              i32(self.spans.start), i32(self.spans.end), i32(self.spans.groups))
+            self.k_pre, self.v_pre = W.make_prefill(w, device)
+            self.q, self.kn, self.vn, self.npos = W.make_steps(w, device)
+            self.out = torch.empty(w.steps, w.layers, w.batch, w.q_heads, w.head_dim, dtype=w.dtype, device=device)
         cap = (w.capacity + 63) // 64 * 64 if paged else w.capacity
         self.desc = CacheDesc(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, cap, w.dtype)
         # a paged pool as large as the dense cache: the footprint reported is the pages in use
         self.pages = w.units * (cap // 64) if paged else None
         self.sess = Session(self.desc, w.budget, w.gamma, sink=w.sink, recent_frac=w.recent_frac,
-                            compaction=compaction, device=device, pages=self.pages)
+                            compaction=compaction, device=device, pages=self.pages,
+                            cache=None if share is None else share.sess.cache)
         self.graph = None
-        self.out = torch.empty(w.steps, w.layers, w.batch, w.q_heads, w.head_dim, dtype=w.dtype, device=device)
 
     def capture(self):
         """Captures the decode loop twice after a stage 1: `graph` as it runs (back-to-back launches,
@@ -320,6 +331,260 @@ def moved_rows(pos_before, n_before, pos_after, n_after):
     shrank = na < nb
     moved = torch.where(shrank, differs.sum(1), torch.zeros_like(na))
     return nb[shrank].cpu().numpy(), moved.cpu().numpy()
+
+
+# ----------------------------------------------------------------------------- target points
+
+# The four target points: the 60-min and 10-min audio workloads, each at the 20x and 4x budgets.
+TARGETS = (("60-min 20x", "stress"), ("60-min 4x", "stress_4x"), ("10-min 20x", "long"), ("10-min 4x", "long_4x"))
+TARGET_FRAC = 0.70
+
+
+class _Flush:
+    """A read-only pass over 1 GiB (torch's sum): evicts L2 without leaving dirty lines behind."""
+
+    def __init__(self, device):
+        self.buf = torch.empty(256 << 20, dtype=torch.float32, device=device)
+        self.out = torch.empty((), dtype=torch.float32, device=device)
+
+    def __call__(self):
+        torch.sum(self.buf, dim=(0,), out=self.out)
+
+
+def _graph_replay_ms(body, reps=3):
+    """Captures `body` once (after one eager run that sets up plans and tensor maps) and returns the
+    replay times in ms (the first replay is a warm-up)."""
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        body()
+    torch.cuda.current_stream().wait_stream(s)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g):
+        body()
+    out = []
+    for r in range(reps + 1):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record()
+        g.replay()
+        e1.record()
+        torch.cuda.synchronize()
+        if r:
+            out.append(e0.elapsed_time(e1))
+    return out, g
+
+
+def _steady_cache(w, n, extra, device, seed=7):
+    """A dense cache of workload w's shape with every unit at length n: seeded N(0, 1) K and V rows,
+    uniform scores, positions in time order (the state the request loop keeps after evictions)."""
+    from paper_2608_08569_gb300 import CacheDesc, allocate_cache
+    desc = CacheDesc(w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, n + extra, w.dtype)
+    c = allocate_cache(desc, device)
+    g = torch.Generator(device=device)
+    g.manual_seed(seed)
+    for b in range(w.batch):
+        c["k"][b].normal_(generator=g)
+        c["v"][b].normal_(generator=g)
+    c["score"].uniform_(generator=g)
+    c["pos"].copy_(torch.arange(desc.capacity, dtype=torch.int32, device=device).expand_as(c["pos"]))
+    c["len"].fill_(n)
+    return desc, c
+
+
+def _frac(nbytes, us, peak):
+    gbs = nbytes / us / 1e3
+    return {"achieved": round(gbs, 1), "frac": round(gbs / peak, 4), "avg_launch_us": round(us, 2)}
+
+
+def flushed_decode(w, r, device, peak, flush, NL=8):
+    """The decode kernel alone at the workload's mean steady-state length (budget + interval / 2),
+    each launch after an L2 flush; median over the launches of two graph replays."""
+    from paper_2608_08569_gb300 import voxzip_decode_step, voxzip_get_status
+    n = max(w.budget) + w.interval // 2
+    desc, c = _steady_cache(w, n, 64, device)
+    q, kn, vn, npos, out = r.q[0], r.kn[0], r.vn[0], r.npos[0], r.out[0]
+    evs = [(torch.cuda.Event(enable_timing=True, external=True), torch.cuda.Event(enable_timing=True, external=True))
+           for _ in range(NL)]
+
+    def body():
+        for a, b in evs:
+            c["len"].fill_(n)
+            flush()
+            a.record()
+            voxzip_decode_step(desc, 0, w.layers, q, kn, vn, npos, c["k"], c["v"], c["score"], c["pos"], c["len"],
+                               w.gamma, out, max_len=n + 1)
+            b.record()
+    times = []
+    _, g = _graph_replay_ms(body, reps=1)
+    for _ in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        times += [a.elapsed_time(b) for a, b in evs]
+    if voxzip_get_status() != 0:
+        raise RuntimeError("device status word set by the flushed decode")
+    us = statistics.median(times) * 1000.0
+    res = _frac(decode_bytes(w, [n + 1] * w.batch), us, peak)
+    res["n"] = n + 1
+    del c, g
+    return res
+
+
+def flushed_evict(w, device, peak, flush, fill=False, NL=6):
+    """The eviction kernel alone at the workload's steady state (budget + interval rows per unit,
+    uniform scores), each launch after restoring that state and an L2 flush."""
+    from paper_2608_08569_gb300 import voxzip_evict, voxzip_evict_ex, voxzip_get_status
+    n = max(w.budget) + w.interval
+    desc, c = _steady_cache(w, n, 64, device, seed=8)
+    ref = {k: v.clone() for k, v in c.items()}
+    bud = torch.tensor(w.budget, dtype=torch.int32, device=device)
+    evs = [(torch.cuda.Event(enable_timing=True, external=True), torch.cuda.Event(enable_timing=True, external=True))
+           for _ in range(NL)]
+
+    def launch():
+        if fill:
+            voxzip_evict_ex(desc, 0, w.layers, c["k"], c["v"], c["score"], c["pos"], c["len"], bud, sink=w.sink,
+                            recent_frac=w.recent_frac, compaction="fill")
+        else:
+            voxzip_evict(desc, 0, w.layers, c["k"], c["v"], c["score"], c["pos"], c["len"], bud, sink=w.sink,
+                         recent_frac=w.recent_frac)
+
+    def body():
+        for a, b in evs:
+            for k in c:
+                c[k].copy_(ref[k])
+            flush()
+            a.record()
+            launch()
+            b.record()
+    times = []
+    _, g = _graph_replay_ms(body, reps=1)
+    for _ in range(2):
+        g.replay()
+        torch.cuda.synchronize()
+        times += [a.elapsed_time(b) for a, b in evs]
+    for k in c:                       # one more, untimed: the rows that changed slot
+        c[k].copy_(ref[k])
+    launch()
+    torch.cuda.synchronize()
+    if voxzip_get_status() != 0:
+        raise RuntimeError("device status word set by the flushed eviction")
+    nb, mv = moved_rows(ref["pos"], ref["len"], c["pos"], c["len"])
+    us = statistics.median(times) * 1000.0
+    res = _frac(evict_bytes(w, nb, mv), us, peak)
+    res["n_before"] = n
+    del c, ref, g
+    return res
+
+
+def decode_loop(w, r, device, NL=32):
+    """Back-to-back decode launches from one CUDA graph (each a programmatic dependent of the one
+    before, no flush: the cache stays in L2 when it fits, as in a serving loop), against the same
+    loop of plain streaming reads of the same bytes (voxzip_stream_read): the most a loop of
+    launches of that size reaches. Starts at the budget, as after an eviction."""
+    from paper_2608_08569_gb300 import voxzip_decode_step, voxzip_get_status, voxzip_stream_read
+    n0 = max(w.budget)
+    desc, c = _steady_cache(w, n0, NL + 64, device, seed=9)
+    q, kn, vn, npos, out = r.q[0], r.kn[0], r.vn[0], r.npos[0], r.out[0]
+
+    def dec():
+        c["len"].fill_(n0)
+        for k in range(NL):
+            voxzip_decode_step(desc, 0, w.layers, q, kn, vn, npos, c["k"], c["v"], c["score"], c["pos"], c["len"],
+                               w.gamma, out, max_len=n0 + k + 1)
+    nbytes = sum(decode_bytes(w, [n0 + k + 1] * w.batch) for k in range(NL)) / NL
+    nb16 = int(nbytes) // 16 * 16
+    buf = torch.empty(nb16 // 4, dtype=torch.int32, device=device).random_(1 << 30)
+    sink = torch.zeros(1, dtype=torch.int32, device=device)
+
+    def rd():
+        c["len"].fill_(n0)
+        for _ in range(NL):
+            voxzip_stream_read(buf, nb16, sink)
+    t_dec = statistics.median(_graph_replay_ms(dec)[0]) * 1000.0 / NL
+    if voxzip_get_status() != 0:
+        raise RuntimeError("device status word set by the decode loop")
+    t_rd = statistics.median(_graph_replay_ms(rd)[0]) * 1000.0 / NL
+    del c, buf
+    return {"us_per_step": round(t_dec, 2), "gbs": round(nbytes / t_dec / 1e3, 1),
+            "read_us_per_step": round(t_rd, 2), "read_gbs": round(nbytes / t_rd / 1e3, 1),
+            "frac_of_read": round(t_rd / t_dec, 4), "launches": NL, "n_start": n0 + 1}
+
+
+def request_view(r, peak, reps=2):
+    """The decode and evict kernels as they run in the workload's request (stage 1, then the decode
+    loop replayed from the instrumented CUDA graph, events around every launch, no flush)."""
+    w = r.w
+    lengths, moved = [], []
+    r.request(lengths=lengths)
+    r.request(moved=moved)
+    torch.cuda.synchronize()
+    r.capture()
+    dec_t, ev_t = [], []
+    for _ in range(reps):
+        r.sess.prefill(r.k_pre, r.v_pre, *r.span_args[:3], *r.span_args[3:])
+        r.graph_timed.replay()
+        torch.cuda.synchronize()
+        dec_t += [a.elapsed_time(b) for kind, a, b in r.graph_events if kind == "decode"]
+        ev_t += [a.elapsed_time(b) for kind, a, b in r.graph_events if kind == "evict"]
+    dec_lens = [n for kind, n in lengths if kind == "decode"]
+    dec_bytes = sum(decode_bytes(w, n) for n in dec_lens) * reps
+    ev_bytes = sum(evict_bytes(w, nb, mv) for nb, mv in moved) * reps
+    dec = _frac(dec_bytes / len(dec_t), 1000.0 * sum(dec_t) / len(dec_t), peak)
+    ev = _frac(ev_bytes / max(1, len(ev_t)), 1000.0 * sum(ev_t) / max(1, len(ev_t)), peak)
+    r.graph = r.graph_timed = None
+    r.graph_events = []
+    return dec, ev
+
+
+def targets_leg(main, device, peak, compaction="ordered", main_request=None):
+    """Decode and eviction against the measured HBM peak at the four target points, three ways:
+    `request` as the workload's request runs them, `flushed` one launch at a time after an L2 flush
+    (the HBM-bound number), `loop` back-to-back launches against a plain read of the same bytes."""
+    from paper_2608_08569_gb300 import workloads as W
+    flush = _Flush(device)
+    runners = {"stress": main}
+    res = {}
+    for label, name in TARGETS:
+        w = W.CONFIGS[name]
+        if name == "stress" and main.w.name == "stress":
+            r = main
+        elif name == "stress_4x" and main.w.name == "stress":
+            r = Runner(w, device, compaction=compaction, share=main)
+        elif name == "long_4x" and "long" in runners:
+            r = Runner(w, device, compaction=compaction, share=runners["long"])
+        else:
+            r = Runner(w, device, compaction=compaction)
+        runners[name] = r
+        if r is main and main_request is not None:   # the timed region above measured this one
+            keys = ("achieved", "frac", "avg_launch_us")
+            dec_req = {k: main_request[0][k] for k in keys}
+            ev_req = {k: main_request[1][k] for k in keys} if main_request[1] else None
+        else:
+            r.request()   # warm-up
+            dec_req, ev_req = request_view(r, peak)
+        res[label] = {
+            "workload": name, "budget": max(w.budget),
+            "decode": {"request": dec_req, "flushed": flushed_decode(w, r, device, peak, flush),
+                       "loop": decode_loop(w, r, device)},
+            "evict": {"request": ev_req, "flushed": flushed_evict(w, device, peak, flush,
+                                                                  fill=compaction == "fill")},
+        }
+        torch.cuda.empty_cache()
+    del runners
+    res["how"] = {
+        "request": "the workload's request (stage 1 + every decode step + evictions) replayed from the "
+                   "instrumented CUDA graph, CUDA events around every launch, L2 not flushed (a 10-min "
+                   "cache of 43-203 MB stays partly in L2 between launches); algorithmic bytes from the "
+                   "request's lengths and moved rows",
+        "flushed": "one launch at a time at the steady state (decode: budget + interval/2 rows per unit; "
+                   "evict: budget + interval), a read-only 1 GiB pass before each launch, median of 12-16 "
+                   "launches: the HBM-bound number",
+        "loop": "32 decode launches back to back from one CUDA graph (programmatic dependent launches, no "
+                "flush), against the same loop of plain streaming reads of the same bytes "
+                "(voxzip_stream_read); frac_of_read = read time / decode time",
+        "target": f">= {TARGET_FRAC} of the measured HBM peak ({peak} GB/s)"}
+    return res
 
 
 def gpu_arm(args, rank, world, local):
@@ -422,6 +687,12 @@ def gpu_arm(args, rank, world, local):
     if not args.no_e2e:
         e2e = e2e_leg(r, args)
     clocks = clk.summary()
+    targets = None
+    if not args.no_targets and not args.paged and w.name == "stress":
+        with ClockSampler(local) as tclk:
+            targets = targets_leg(r, dev, peak, compaction=args.compaction,
+                                  main_request=(roofline, roofline_evict))
+        targets["clocks"] = tclk.summary()
     result = {
         "metric": METRIC, "value": round(value, 2), "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": round(ms_max / args.steps, 3), "higher_is_better": True,
@@ -448,7 +719,7 @@ def gpu_arm(args, rank, world, local):
                    "parallelism": f"replicas x{world} (independent units, no collective)",
                    "l2": "inputs larger than L2 (decode reads ~0.9-7 GB per launch, L2 is 129 MB)"},
         "roofline": roofline, "roofline_evict": roofline_evict, "gpu_launches": gpu_launches, "clocks": clocks,
-        "e2e": e2e,
+        "e2e": e2e, "targets": targets,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         result["cpu_baseline"] = cpu_sample(w, args.cpu_units, compaction=args.compaction)
