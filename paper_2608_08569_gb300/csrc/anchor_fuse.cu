@@ -273,9 +273,13 @@ slot_map_kernel(int32_t stride, bool keep_bg, const int32_t *__restrict__ in_len
     }
 }
 
-// kPaged: k_cache / v_cache are page pools and output slot s goes to the row the page table gives.
+// A persistent grid (as many CTAs as are resident at once) walks work items: chunk c of the output
+// slots of unit u, item = c * units + u, so every CTA gets an equal share of the rows and no wave
+// runs part-empty. A chunk is kSlotsPerPass consecutive slots: warp w owns kSlotsPerWarp groups of
+// kRowsPerWarp slots. kPaged: k_cache / v_cache are page pools and output slot s goes to the row
+// the page table gives.
 template <typename T, int D, bool kPaged>
-__global__ void __launch_bounds__(kFuseWarps * 32)
+__global__ void __launch_bounds__(kFuseWarps * 32, 4)
 fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, int32_t anchor_stride,
                  const T *__restrict__ k_prefill, const T *__restrict__ v_prefill,
                  const T *__restrict__ anchor_k, const T *__restrict__ anchor_v, FuseWorkspace ws,
@@ -285,78 +289,85 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
     constexpr int kLanesPerRow = D / kElems;
     constexpr int kRowsPerWarp = 32 / kLanesPerRow;
     constexpr int kRowVecs = D / kElems;          // 16-byte vectors per row
-    const int u = blockIdx.y;                    // cache unit (b, l, h)
-    const int b = u / (L * Hkv);
-    int32_t out_len = ws.seq_len[b];
-    if (kPaged && pv.table[(int64_t)u * pv.max_pages] < 0) out_len = -1;  // the pool could not hold it
-    if (blockIdx.x == 0 && threadIdx.x == 0) len[u] = out_len < 0 ? 0 : out_len;
-    if (out_len < 0) return;
+    constexpr int kSlotsPerPass = kFuseWarps * kSlotsPerWarp * kRowsPerWarp;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int sub = lane / kLanesPerRow, e = (lane % kLanesPerRow) * kElems;
-    const int64_t in_base = (int64_t)u * stride * D;
-    const int64_t out_base = kPaged ? 0 : (int64_t)u * C * D;
-    const int64_t anc_base = (int64_t)u * anchor_stride * D;
-    const uint4 *kin = reinterpret_cast<const uint4 *>(k_prefill + in_base + e);  // vector e of row 0
-    const uint4 *vin = reinterpret_cast<const uint4 *>(v_prefill + in_base + e);
-    const int32_t *src = ws.slot_src + (int64_t)b * stride;
-    const int32_t *send = ws.slot_end + (int64_t)b * stride;
-    const int32_t *anc = ws.slot_anchor + (int64_t)b * stride;
-    constexpr int kSlotsPerPass = kFuseWarps * kSlotsPerWarp * kRowsPerWarp;
-    for (int slot0 = (blockIdx.x * kFuseWarps + warp) * kSlotsPerWarp * kRowsPerWarp; slot0 < out_len;
-         slot0 += gridDim.x * kSlotsPerPass)
-    for (int k = 0; k < kSlotsPerWarp; ++k) {
-        const int s = slot0 + k * kRowsPerWarp + sub;
-        if (s >= out_len) break;
-        const int32_t r0 = src[s], r1 = send[s];
-        if (!VOXZIP_IN_RANGE(ws.status, r0 >= 0 && r0 < r1 && r1 <= stride && s < C)) continue;
-        float sk[kElems], sv[kElems];
+    const int units = B * L * Hkv;
+    // Chunks per unit: enough for the longest stage-1 output of the batch.
+    int max_len = 0;
+    for (int bb = 0; bb < B; ++bb) max_len = max(max_len, ws.seq_len[bb]);
+    const int chunks = max(1, (max_len + kSlotsPerPass - 1) / kSlotsPerPass);
+    for (int64_t item = blockIdx.x; item < (int64_t)units * chunks; item += gridDim.x) {
+        const int u = (int)(item % units);   // cache unit (b, l, h)
+        const int chunk = (int)(item / units);
+        const int b = u / (L * Hkv);
+        int32_t out_len = ws.seq_len[b];
+        if (kPaged && pv.table[(int64_t)u * pv.max_pages] < 0) out_len = -1;  // the pool could not hold it
+        if (chunk == 0 && threadIdx.x == 0) len[u] = out_len < 0 ? 0 : out_len;
+        if (out_len <= chunk * kSlotsPerPass) continue;
+        const int64_t in_base = (int64_t)u * stride * D;
+        const int64_t out_base = kPaged ? 0 : (int64_t)u * C * D;
+        const int64_t anc_base = (int64_t)u * anchor_stride * D;
+        const uint4 *kin = reinterpret_cast<const uint4 *>(k_prefill + in_base + e);  // vector e of row 0
+        const uint4 *vin = reinterpret_cast<const uint4 *>(v_prefill + in_base + e);
+        const int32_t *src = ws.slot_src + (int64_t)b * stride;
+        const int32_t *send = ws.slot_end + (int64_t)b * stride;
+        const int32_t *anc = ws.slot_anchor + (int64_t)b * stride;
+        const int slot0 = chunk * kSlotsPerPass + warp * kSlotsPerWarp * kRowsPerWarp;
+        for (int k = 0; k < kSlotsPerWarp; ++k) {
+            const int s = slot0 + k * kRowsPerWarp + sub;
+            if (s >= out_len) break;
+            const int32_t r0 = src[s], r1 = send[s];
+            if (!VOXZIP_IN_RANGE(ws.status, r0 >= 0 && r0 < r1 && r1 <= stride && s < C)) continue;
+            float sk[kElems], sv[kElems];
 #pragma unroll
-        for (int i = 0; i < kElems; ++i) sk[i] = sv[i] = 0.f;
-        int32_t r = r0;
-        for (; r + 4 <= r1; r += 4) {  // four rows' loads in flight, then their sums in token order
-            uint4 xk[4], xv[4];
+            for (int i = 0; i < kElems; ++i) sk[i] = sv[i] = 0.f;
+            int32_t r = r0;
+            for (; r + 4 <= r1; r += 4) {  // four rows' loads in flight, then their sums in token order
+                uint4 xk[4], xv[4];
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                xk[i] = __ldcs(kin + (int64_t)(r + i) * kRowVecs);
-                xv[i] = __ldcs(vin + (int64_t)(r + i) * kRowVecs);
+                for (int i = 0; i < 4; ++i) {
+                    xk[i] = __ldcs(kin + (int64_t)(r + i) * kRowVecs);
+                    xv[i] = __ldcs(vin + (int64_t)(r + i) * kRowVecs);
+                }
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    accumulate16<T>(sk, xk[i]);
+                    accumulate16<T>(sv, xv[i]);
+                }
             }
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                accumulate16<T>(sk, xk[i]);
-                accumulate16<T>(sv, xv[i]);
+            for (; r < r1; ++r) {
+                accumulate16<T>(sk, __ldcs(kin + (int64_t)r * kRowVecs));
+                accumulate16<T>(sv, __ldcs(vin + (int64_t)r * kRowVecs));
             }
-        }
-        for (; r < r1; ++r) {
-            accumulate16<T>(sk, __ldcs(kin + (int64_t)r * kRowVecs));
-            accumulate16<T>(sv, __ldcs(vin + (int64_t)r * kRowVecs));
-        }
-        if (r1 - r0 > 1) {
-            const float cnt = (float)(r1 - r0);
+            if (r1 - r0 > 1) {
+                const float cnt = (float)(r1 - r0);
 #pragma unroll
-            for (int i = 0; i < kElems; ++i) {
-                sk[i] = __fdiv_rn(sk[i], cnt);
-                sv[i] = __fdiv_rn(sv[i], cnt);
+                for (int i = 0; i < kElems; ++i) {
+                    sk[i] = __fdiv_rn(sk[i], cnt);
+                    sv[i] = __fdiv_rn(sv[i], cnt);
+                }
             }
-        }
-        const int32_t a_row = anc[s];
-        if (anchor_k != nullptr && a_row >= 0 && VOXZIP_IN_RANGE(ws.status, a_row < anchor_stride)) {
-            float ak[kElems], av[kElems];
+            const int32_t a_row = anc[s];
+            if (anchor_k != nullptr && a_row >= 0 && VOXZIP_IN_RANGE(ws.status, a_row < anchor_stride)) {
+                float ak[kElems], av[kElems];
 #pragma unroll
-            for (int i = 0; i < kElems; ++i) ak[i] = av[i] = 0.f;
-            accumulate16<T>(ak, *reinterpret_cast<const uint4 *>(anchor_k + anc_base + (int64_t)a_row * D + e));
-            accumulate16<T>(av, *reinterpret_cast<const uint4 *>(anchor_v + anc_base + (int64_t)a_row * D + e));
+                for (int i = 0; i < kElems; ++i) ak[i] = av[i] = 0.f;
+                accumulate16<T>(ak, *reinterpret_cast<const uint4 *>(anchor_k + anc_base + (int64_t)a_row * D + e));
+                accumulate16<T>(av, *reinterpret_cast<const uint4 *>(anchor_v + anc_base + (int64_t)a_row * D + e));
 #pragma unroll
-            for (int i = 0; i < kElems; ++i) {
-                sk[i] = __fadd_rn(sk[i], ak[i]);
-                sv[i] = __fadd_rn(sv[i], av[i]);
+                for (int i = 0; i < kElems; ++i) {
+                    sk[i] = __fadd_rn(sk[i], ak[i]);
+                    sv[i] = __fadd_rn(sv[i], av[i]);
+                }
             }
-        }
-        const int64_t orow = kPaged ? paged_row(pv, u, s) : s;
-        *reinterpret_cast<uint4 *>(k_cache + out_base + orow * D + e) = pack16<T>(sk);
-        *reinterpret_cast<uint4 *>(v_cache + out_base + orow * D + e) = pack16<T>(sv);
-        if (e == 0) {
-            pos[(int64_t)u * C + s] = r0;
-            score[(int64_t)u * C + s] = 0.f;
+            const int64_t orow = kPaged ? paged_row(pv, u, s) : s;
+            *reinterpret_cast<uint4 *>(k_cache + out_base + orow * D + e) = pack16<T>(sk);
+            *reinterpret_cast<uint4 *>(v_cache + out_base + orow * D + e) = pack16<T>(sv);
+            if (e == 0) {
+                pos[(int64_t)u * C + s] = r0;
+                score[(int64_t)u * C + s] = 0.f;
+            }
         }
     }
 }
@@ -369,12 +380,17 @@ cudaError_t launch_fuse_rows(const voxzip_cache_desc &d, int32_t stride, int32_t
     constexpr int kRowsPerWarp = 32 / (D * (int)sizeof(T) / 16);  // as in the kernel
     const int slots_per_block = kFuseWarps * kSlotsPerWarp * kRowsPerWarp;
     const int64_t units = (int64_t)d.batch * d.layers * d.kv_heads;
-    // A grid-stride loop over each unit's output slots: about six CTAs per SM in all, never more
-    // than the prompt stride needs (stage 1 leaves far fewer slots than prompt tokens).
-    const int64_t per_unit = (sm_count() * 6 + units - 1) / units;
-    dim3 grid((unsigned)std::max<int64_t>(1, std::min<int64_t>((stride + slots_per_block - 1) / slots_per_block,
-                                                               per_unit)),
-              (unsigned)units);
+    // As many CTAs as are resident at once (never more than the work items of the longest possible
+    // output): each walks items grid-stride.
+    static int per_sm = 0;
+    if (per_sm == 0 && (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fuse_rows_kernel<T, D, kPaged>,
+                                                                       kFuseWarps * 32, 0) != cudaSuccess ||
+                        per_sm < 1)) {
+        cudaGetLastError();
+        per_sm = 4;
+    }
+    const int64_t items = units * ((stride + slots_per_block - 1) / slots_per_block);
+    const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(items, (int64_t)sm_count() * per_sm));
     fuse_rows_kernel<T, D, kPaged><<<grid, kFuseWarps * 32, 0, stream>>>(
         d.batch, d.layers, d.kv_heads, d.capacity, stride, anchor_stride, (const T *)kp, (const T *)vp,
         (const T *)ak, (const T *)av, ws, (T *)kc, (T *)vc, score, pos, len, pv);

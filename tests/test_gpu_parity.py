@@ -42,8 +42,11 @@ def _pipeline(w, sample_k, steps=None, anchors=False):
     st = check_units.last_stats
     print(f"\n[parity] {w.name}: {len(sample)} units, {st['evictions']} evictions compared, "
           f"max |out err| {st['max_out_err']:.3g}, max score rel err {st['max_score_rel']:.3g}, "
-          f"diverged at near-ties: {diverged}")
-    assert len(diverged) <= max(1, len(sample) // 4), diverged
+          f"{len(diverged)} unit(s) left at a near-tie: {diverged}")
+    # A unit leaves the comparison only when the two kept sets differ at an eviction whose N-th vs
+    # (N+1)-th score margin is within the score tolerance (Eq. 9's tie rule, reading R12). The GPU's
+    # fp32 error (~1e-6 relative) flips such an order rarely: at most one unit in eight may leave.
+    assert len(diverged) <= max(1, len(sample) // 8), diverged
     return rec, res, diverged
 
 
@@ -67,8 +70,10 @@ def test_whole_path_with_anchors():
 
 
 @pytest.mark.parametrize("name,k,steps", [("long", 24, None), ("long_4x", 12, None), ("batched", 16, None),
-                                          ("stress", 6, None), ("stress_4x", 3, 96)])
+                                          ("stress", 12, None), ("stress_4x", 6, None)])
 def test_full_size_sampled_units(name, k, steps):
+    """Whole requests at full size (all 48 layers, every sequence, every decode step and eviction on
+    the GPU); the oracle follows a seeded sample of k units through the same request."""
     w = W.CONFIGS[name]
     _pipeline(w, sample_k=k, steps=steps)
 
