@@ -744,18 +744,31 @@ struct Plan {
 
 struct PlanModel {
     double cta_fixed_us, cluster_fixed_us, stage_tokens_per_us, sm_tokens_per_us, gpu_tokens_per_us;
+    int stage_cap;  // ring stages beyond this add no streaming rate
 };
+// A launch whose K and V stream from HBM.
 constexpr PlanModel kPlanModel{VOXZIP_DECODE_CTA_FIXED_US, VOXZIP_DECODE_CLUSTER_FIXED_US,
                                VOXZIP_DECODE_STAGE_TOKENS_PER_US, VOXZIP_DECODE_SM_TOKENS_PER_US,
-                               VOXZIP_DECODE_GPU_TOKENS_PER_US};
+                               VOXZIP_DECODE_GPU_TOKENS_PER_US, 8};
+// A launch whose K and V fit comfortably in L2 (at most VOXZIP_DECODE_L2_RESIDENT_MB): in a decode
+// loop they stay there from step to step. Fitted to back-to-back graph loops on GB300 (10-min and
+// 30-s requests, cluster sizes 1-4, ring depths 2-4): a CTA then consumes ~46 tokens/us whatever
+// its ring depth past three stages, an SM ~120, and a cluster exchange adds ~2.6 us.
+constexpr PlanModel kPlanModelL2{VOXZIP_DECODE_CTA_FIXED_US, 2.6, 46.0 / 3.0, 120.0, 30000.0, 3};
+#ifndef VOXZIP_DECODE_L2_RESIDENT_MB
+#define VOXZIP_DECODE_L2_RESIDENT_MB 64.0
+#endif
 
 // Chooses the cluster size S and ring depth NS with a time model. For each (S, NS) the CTAs hold
 // ceil(nmax/S) tokens (shared memory sized for that, rounded up to 16 tokens); the occupancy API
 // gives how many clusters are resident. Every resident cluster takes ceil(units / clusters) units
 // in turn; a unit costs a CTA's fixed latency (more with a cluster exchange) plus its tokens at one
 // CTA's streaming rate, which grows with the ring stages in flight until the CTAs resident on an SM
-// share its bandwidth; and no launch beats the GPU's streaming rate.
-Plan plan(int D, int NT, int units, int nmax, bool paged = false, const PlanModel &md = kPlanModel) {
+// share its bandwidth; and no launch beats the GPU's streaming rate. A launch small enough to stay
+// in L2 across a decode loop is planned with the L2 constants instead.
+Plan plan(int D, int NT, int units, int nmax, bool paged = false) {
+    const bool l2 = (double)units * nmax * 4.0 * D <= VOXZIP_DECODE_L2_RESIDENT_MB * 1048576.0;
+    const PlanModel &md = l2 ? kPlanModelL2 : kPlanModel;
     Plan best{0, 3, 0};
     double best_cost = 0.0;
     int sms = 148;
@@ -777,7 +790,7 @@ Plan plan(int D, int NT, int units, int nmax, bool paged = false, const PlanMode
             const int cl = dispatch(D, NT, ns, [&](auto k) { return max_active_clusters<decltype(k)>(S, sm); });
             if (cl <= 0) continue;
             const double per_sm = fmax(1.0, (double)min(units, cl) * S / sms);  // CTAs sharing an SM
-            const double rate = fmin(md.stage_tokens_per_us * ns, md.sm_tokens_per_us / per_sm);
+            const double rate = fmin(md.stage_tokens_per_us * min(ns, md.stage_cap), md.sm_tokens_per_us / per_sm);
             const double rounds = (double)((units + cl - 1) / cl);
             const double per_cta = md.cta_fixed_us + (S > 1 ? md.cluster_fixed_us : 0.0) +
                                    (double)((nmax + S - 1) / S) / rate;
