@@ -96,7 +96,12 @@ typedef struct {
  * keep chronological order; pos[slot] = index of the slot's first prefill token; score = 0;
  * len = number of rows, the same for every unit of a sequence.
  *
- *   k_prefill, v_prefill  [B][L][Hkv][prefill_stride][D]; rows [0, in_len[b]) are read
+ *   k_prefill, v_prefill  [B][L][Hkv][prefill_stride][D]; rows [0, in_len[b]) are read, each
+ *                         once. Device memory, or page-locked host memory that the device
+ *                         addresses directly (unified addressing, as across the C2C link of a
+ *                         Grace-Blackwell node): the kernels then stream the rows over the host
+ *                         link from CTAs on half the SMs, need no device copy of the prompt, and
+ *                         leave the other SMs to kernels running beside them.
  *   in_len, audio_begin, audio_len  [B] device int32
  *   span_off              [B+1] device int32, span_off[0] = 0, span_off[B] = num_spans
  *   span_start, span_end, span_groups  [num_spans] device int32

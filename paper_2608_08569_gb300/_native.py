@@ -169,13 +169,15 @@ def _stream(stream):
     return ctypes.c_void_p(s.cuda_stream)
 
 
-def _need(t: torch.Tensor, name: str, dtype: torch.dtype, shape=None) -> None:
+def _need(t: torch.Tensor, name: str, dtype: torch.dtype, shape=None, pinned_ok: bool = False) -> None:
+    """Checks a tensor argument; `pinned_ok` also accepts page-locked host memory (which the device
+    addresses directly under unified addressing)."""
     if not isinstance(t, torch.Tensor):
         raise TypeError(f"{name} must be a torch.Tensor")
     if t.dtype != dtype:
         raise ValueError(f"{name}: dtype {t.dtype}, expected {dtype}")
-    if not t.is_cuda:
-        raise ValueError(f"{name} must be on a CUDA device")
+    if not t.is_cuda and not (pinned_ok and t.is_pinned()):
+        raise ValueError(f"{name} must be on a CUDA device" + (" or in pinned host memory" if pinned_ok else ""))
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
     if shape is not None and tuple(t.shape) != tuple(shape):
@@ -259,8 +261,8 @@ def voxzip_anchor_fuse_paged(desc: CacheDesc, pc, k_prefill, v_prefill, in_len, 
     stage-1 rows need."""
     B, L, H, D = desc.batch, desc.layers, desc.kv_heads, desc.head_dim
     stride = k_prefill.shape[3]
-    _need(k_prefill, "k_prefill", desc.dtype, (B, L, H, stride, D))
-    _need(v_prefill, "v_prefill", desc.dtype, (B, L, H, stride, D))
+    _need(k_prefill, "k_prefill", desc.dtype, (B, L, H, stride, D), pinned_ok=True)
+    _need(v_prefill, "v_prefill", desc.dtype, (B, L, H, stride, D), pinned_ok=True)
     for name, t in (("in_len", in_len), ("audio_begin", audio_begin), ("audio_len", audio_len)):
         _need(t, name, torch.int32, (B,))
     _need(span_off, "span_off", torch.int32, (B + 1,))
@@ -339,8 +341,8 @@ def voxzip_anchor_fuse(desc: CacheDesc, k_prefill, v_prefill, in_len, audio_begi
     if k_prefill.dim() != 5:
         raise ValueError("k_prefill must be [B][L][Hkv][stride][D]")
     stride = k_prefill.shape[3]
-    _need(k_prefill, "k_prefill", desc.dtype, (B, L, H, stride, D))
-    _need(v_prefill, "v_prefill", desc.dtype, (B, L, H, stride, D))
+    _need(k_prefill, "k_prefill", desc.dtype, (B, L, H, stride, D), pinned_ok=True)
+    _need(v_prefill, "v_prefill", desc.dtype, (B, L, H, stride, D), pinned_ok=True)
     for name, t in (("in_len", in_len), ("audio_begin", audio_begin), ("audio_len", audio_len)):
         _need(t, name, torch.int32, (B,))
     _need(span_off, "span_off", torch.int32, (B + 1,))
@@ -441,8 +443,8 @@ def voxzip_anchor_fuse_noalloc(desc: CacheDesc, k_prefill, v_prefill, in_len, au
     if k_prefill.dim() != 5:
         raise ValueError("k_prefill must be [B][L][Hkv][stride][D]")
     stride = k_prefill.shape[3]
-    _need(k_prefill, "k_prefill", desc.dtype, (B, L, H, stride, D))
-    _need(v_prefill, "v_prefill", desc.dtype, (B, L, H, stride, D))
+    _need(k_prefill, "k_prefill", desc.dtype, (B, L, H, stride, D), pinned_ok=True)
+    _need(v_prefill, "v_prefill", desc.dtype, (B, L, H, stride, D), pinned_ok=True)
     for name, t in (("in_len", in_len), ("audio_begin", audio_begin), ("audio_len", audio_len)):
         _need(t, name, torch.int32, (B,))
     _need(span_off, "span_off", torch.int32, (B + 1,))

@@ -78,6 +78,10 @@ __device__ __forceinline__ uint4 pack16<__nv_bfloat16>(const float *acc) {
     return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
+#ifndef VOXZIP_FUSE_HOST_CTAS
+#define VOXZIP_FUSE_HOST_CTAS 0  // stage-1 CTAs when the prefill rows are in host memory (0: half the SMs)
+#endif
+
 constexpr int kScanThreads = 512;
 constexpr int kMapThreads = 256;
 constexpr int kFuseWarps = 8;
@@ -390,7 +394,17 @@ cudaError_t launch_fuse_rows(const voxzip_cache_desc &d, int32_t stride, int32_t
         per_sm = 4;
     }
     const int64_t items = units * ((stride + slots_per_block - 1) / slots_per_block);
-    const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(items, (int64_t)sm_count() * per_sm));
+    // Prefill rows in host memory the device addresses directly (page-locked memory under unified
+    // addressing, across the Grace-Blackwell C2C link): the kernel streams them over the host link.
+    // CTAs on half the SMs already keep the link busy (on GB300: 87 ms for the 18.1 GB of a 60-min
+    // request, ~209 GB/s), and the rest of the GPU stays free for a kernel running beside it: a decode
+    // loop of another request slows by ~2% (by 67% when every SM also runs a stage-1 CTA).
+    cudaPointerAttributes pa{};
+    const bool host_rows = cudaPointerGetAttributes(&pa, kp) == cudaSuccess && pa.type == cudaMemoryTypeHost;
+    cudaGetLastError();
+    const int64_t ctas = host_rows ? (VOXZIP_FUSE_HOST_CTAS > 0 ? VOXZIP_FUSE_HOST_CTAS : std::max(1, sm_count() / 2))
+                                   : (int64_t)sm_count() * per_sm;
+    const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(items, ctas));
     fuse_rows_kernel<T, D, kPaged><<<grid, kFuseWarps * 32, 0, stream>>>(
         d.batch, d.layers, d.kv_heads, d.capacity, stride, anchor_stride, (const T *)kp, (const T *)vp,
         (const T *)ak, (const T *)av, ws, (T *)kc, (T *)vc, score, pos, len, pv);

@@ -42,6 +42,13 @@ namespace voxzip {
 namespace {
 
 constexpr int kThreads = 256;
+// Hole filling runs 256-thread CTAs (4 per SM) when a launch's units fit one wave of those, else
+// 192-thread CTAs (6 per SM: the 768 units of 4 sequences x 48 layers x 4 kv-heads in one wave).
+// Its time is the latency of its radix passes, so fewer waves beat more threads per pass.
+template <int NT>
+struct FillShape {
+    static constexpr int kCtasPerSm = NT <= 192 ? 6 : 4;
+};
 constexpr int kSegment = 1024;   // ranks listed per compaction segment
 constexpr uint32_t kEvictWaitLimit = 1u << 22;  // polls before an mbarrier wait gives up
 
@@ -114,10 +121,11 @@ __device__ __forceinline__ uint32_t score_key(float s) {  // monotone map of fp3
     return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
-// Block-wide exclusive scan of one int per thread.
+// Block-wide exclusive scan of one int per thread (NT threads).
+template <int NT = kThreads>
 __device__ int scan_excl(int v, int *total, int *warp_sums) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    constexpr int kWarps = kThreads / 32;
+    constexpr int kWarps = NT / 32;
     int x = v;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -152,20 +160,13 @@ struct RadixState {
     int bin;
 };
 
-template <bool kDescending, typename KeyFn>
-__device__ void radix_pass(int shift, int lo, int hi, KeyFn key_of, RadixState &st, unsigned *hist,
-                           RadixState *shared_st) {
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    for (int i = tid; i < 256; i += kThreads) hist[i] = 0u;
-    __syncthreads();
-    const uint32_t mask_hi = shift == 24 ? 0u : (0xffffffffu << (shift + 8));
-    for (int j = lo + tid; j < hi; j += kThreads) {
-        bool valid;
-        const uint32_t k = key_of(j, valid);
-        if (valid && (k & mask_hi) == (st.prefix & mask_hi)) atomicAdd(&hist[(k >> shift) & 255u], 1u);
-    }
-    __syncthreads();
-    if (warp == 0) {
+// One warp finds the bin of the rem-th key of a 256-bin histogram, counted from the top bin
+// (descending) or the bottom, and publishes the new prefix, remainder and bin size.
+template <bool kDescending>
+__device__ __forceinline__ void radix_find(int shift, uint32_t mask_hi, const RadixState &st, const unsigned *hist,
+                                           RadixState *shared_st) {
+    const int lane = threadIdx.x & 31;
+    {
         // Lane l holds 8 consecutive bins in scan order (from the top bin when descending).
         unsigned c[8], s = 0;
 #pragma unroll
@@ -197,8 +198,50 @@ __device__ void radix_pass(int shift, int lo, int hi, KeyFn key_of, RadixState &
             }
         }
     }
+}
+
+template <bool kDescending, int NT = kThreads, typename KeyFn>
+__device__ void radix_pass(int shift, int lo, int hi, KeyFn key_of, RadixState &st, unsigned *hist,
+                           RadixState *shared_st) {
+    const int tid = threadIdx.x, warp = tid >> 5;
+    for (int i = tid; i < 256; i += NT) hist[i] = 0u;
+    __syncthreads();
+    const uint32_t mask_hi = shift == 24 ? 0u : (0xffffffffu << (shift + 8));
+    for (int j = lo + tid; j < hi; j += NT) {
+        bool valid;
+        const uint32_t k = key_of(j, valid);
+        if (valid && (k & mask_hi) == (st.prefix & mask_hi)) atomicAdd(&hist[(k >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (warp == 0) radix_find<kDescending>(shift, mask_hi, st, hist, shared_st);
     __syncthreads();
     st = *shared_st;
+}
+
+// Two selects over the same keys in one sweep per digit: `lo_st` counts from the bottom (the
+// rem-th smallest key), `hi_st` from the top, each with its own histogram; warp 0 and warp 1 find
+// their bins at the same time.
+template <int NT, typename KeyFn>
+__device__ void radix_pass_both(int shift, int n, KeyFn key_of, RadixState &lo_st, RadixState &hi_st,
+                                unsigned *hist_lo, unsigned *hist_hi, RadixState *shared_lo, RadixState *shared_hi) {
+    const int tid = threadIdx.x, warp = tid >> 5;
+    for (int i = tid; i < 256; i += NT) hist_lo[i] = hist_hi[i] = 0u;
+    __syncthreads();
+    const uint32_t mask_hi = shift == 24 ? 0u : (0xffffffffu << (shift + 8));
+    for (int j = tid; j < n; j += NT) {
+        bool valid;
+        const uint32_t k = key_of(j, valid);
+        if (!valid) continue;
+        const unsigned bin = (k >> shift) & 255u;
+        if ((k & mask_hi) == (lo_st.prefix & mask_hi)) atomicAdd(&hist_lo[bin], 1u);
+        if ((k & mask_hi) == (hi_st.prefix & mask_hi)) atomicAdd(&hist_hi[bin], 1u);
+    }
+    __syncthreads();
+    if (warp == 0) radix_find<false>(shift, mask_hi, lo_st, hist_lo, shared_lo);
+    if (warp == 1) radix_find<true>(shift, mask_hi, hi_st, hist_hi, shared_hi);
+    __syncthreads();
+    lo_st = *shared_lo;
+    hi_st = *shared_hi;
 }
 
 template <typename T, int D, bool kPaged, bool kWide>
@@ -485,14 +528,14 @@ evict_kernel(const EvictParams p) {
     }
 }
 
-template <typename T, int D, bool kPaged>
-__global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictParams p) {
+template <typename T, int D, bool kPaged, int NT>
+__global__ void __launch_bounds__(NT, FillShape<NT>::kCtasPerSm) evict_fill_kernel(const EvictParams p) {
     constexpr int kVecPerRow = D * (int)sizeof(T) / 16;
     __shared__ int32_t holes[kSegment];
     __shared__ int32_t movers[kSegment];
-    __shared__ unsigned hist[256];
+    __shared__ unsigned hist[256], hist2[256];
     __shared__ int warp_sums[32];
-    __shared__ RadixState shared_st;
+    __shared__ RadixState shared_st, shared_st2;
     __shared__ int resume_at;
     const int tid = threadIdx.x;
     const UnitIdx ui = unit_of(blockIdx.x, p.B, p.L, p.Hkv, p.layer_begin);
@@ -526,25 +569,32 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
     // The bits any position sets: radix passes over high digits that are zero in every position
     // (positions below 2^16, say) decide nothing and are skipped.
     uint32_t any = 0u;
-    for (int j = tid; j < n; j += kThreads) any |= (uint32_t)ps[j];
+    for (int j = tid; j < n; j += NT) any |= (uint32_t)ps[j];
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) any |= __shfl_xor_sync(0xffffffffu, any, o);
     if ((tid & 31) == 0) warp_sums[tid >> 5] = (int)any;
     __syncthreads();
     any = 0u;
 #pragma unroll
-    for (int w = 0; w < kThreads / 32; ++w) any |= (uint32_t)warp_sums[w];
+    for (int w = 0; w < NT / 32; ++w) any |= (uint32_t)warp_sums[w];
     __syncthreads();
     const int top_shift = any >> 24 ? 24 : any >> 16 ? 16 : any >> 8 ? 8 : 0;
     uint32_t p_lo = 0u, p_hi = 0xffffffffu;
-    if (T_ > 0) {
+    if (T_ > 0 && M > 0) {  // both cuts in one sweep per digit
+        RadixState lo{0u, T_, 0}, hi{0u, M, 0};
+        for (int shift = top_shift; shift >= 0; shift -= 8)
+            radix_pass_both<NT>(shift, n, pkey, lo, hi, hist, hist2, &shared_st, &shared_st2);
+        p_lo = lo.prefix;
+        p_hi = hi.prefix;
+    } else if (T_ > 0) {
         RadixState st{0u, T_, 0};
-        for (int shift = top_shift; shift >= 0; shift -= 8) radix_pass<false>(shift, 0, n, pkey, st, hist, &shared_st);
+        for (int shift = top_shift; shift >= 0; shift -= 8)
+            radix_pass<false, NT>(shift, 0, n, pkey, st, hist, &shared_st);
         p_lo = st.prefix;
-    }
-    if (M > 0) {
+    } else if (M > 0) {
         RadixState st{0u, M, 0};
-        for (int shift = top_shift; shift >= 0; shift -= 8) radix_pass<true>(shift, 0, n, pkey, st, hist, &shared_st);
+        for (int shift = top_shift; shift >= 0; shift -= 8)
+            radix_pass<true, NT>(shift, 0, n, pkey, st, hist, &shared_st);
         p_hi = st.prefix;
     }
     auto middle = [&](uint32_t q) { return !(T_ > 0 && q <= p_lo) && !(M > 0 && q >= p_hi); };
@@ -558,7 +608,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
             valid = middle((uint32_t)ps[j]);
             return score_key(sc[j]);
         };
-        for (int shift = 24; shift >= 0; shift -= 8) radix_pass<true>(shift, 0, n, skey, st, hist, &shared_st);
+        for (int shift = 24; shift >= 0; shift -= 8) radix_pass<true, NT>(shift, 0, n, skey, st, hist, &shared_st);
         thr = st.prefix;
         all_ties = st.rem == st.bin;
         if (!all_ties) {
@@ -569,7 +619,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
                 return q;
             };
             for (int shift = top_shift; shift >= 0; shift -= 8)
-                radix_pass<false>(shift, 0, n, tkey, sq, hist, &shared_st);
+                radix_pass<false, NT>(shift, 0, n, tkey, sq, hist, &shared_st);
             pos_thr = sq.prefix;
         }
     }
@@ -586,14 +636,14 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
     int hcur = 0, mcur = bud;
     while (true) {
         int nh = 0;
-        while (hcur < bud && nh + kThreads <= kSegment) {
+        while (hcur < bud && nh + NT <= kSegment) {
             const int j = hcur + tid;
             const bool hole = j < bud && !kept(j);
             int total;
-            const int r = scan_excl(hole ? 1 : 0, &total, warp_sums);
+            const int r = scan_excl<NT>(hole ? 1 : 0, &total, warp_sums);
             if (hole) holes[nh + r] = j;
             nh += total;
-            hcur += kThreads;
+            hcur += NT;
         }
         if (nh == 0) break;
         int nm = 0;
@@ -601,11 +651,11 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
             const int j = mcur + tid;
             const bool mv = j < n && kept(j);
             int total;
-            const int r = scan_excl(mv ? 1 : 0, &total, warp_sums);
+            const int r = scan_excl<NT>(mv ? 1 : 0, &total, warp_sums);
             if (mv && nm + r < nh) movers[nm + r] = j;
             if (nm + total <= nh) {
                 nm += total;
-                mcur += kThreads;
+                mcur += NT;
             } else {  // this step holds more movers than holes are left: resume after the last one taken
                 if (mv && nm + r == nh - 1) resume_at = j + 1;
                 __syncthreads();
@@ -617,7 +667,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
         __syncthreads();
         const int pairs = min(nh, nm);  // equal when positions are unique (then exactly `bud` rows are kept)
         if (pairs < nh && tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_POSITIONS);
-        for (int v = tid; v < pairs * 2 * kVecPerRow; v += kThreads) {
+        for (int v = tid; v < pairs * 2 * kVecPerRow; v += NT) {
             const int r = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
             uint4 *base = w < kVecPerRow ? kc : vc;
             const int e = w % kVecPerRow;
@@ -625,7 +675,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
                                            row_ok(slot_row(holes[r])) && row_ok(slot_row(movers[r]))))
                 base[slot_row(holes[r]) * kVecPerRow + e] = base[slot_row(movers[r]) * kVecPerRow + e];
         }
-        for (int r = tid; r < pairs; r += kThreads) {
+        for (int r = tid; r < pairs; r += NT) {
             sc[holes[r]] = sc[movers[r]];
             ps[holes[r]] = ps[movers[r]];
         }
@@ -635,7 +685,7 @@ __global__ void __launch_bounds__(kThreads, 4) evict_fill_kernel(const EvictPara
     // Every kept row at or above the budget has found a hole; one left over means more than
     // `bud` rows were kept (repeated positions).
     int extra = 0;
-    for (int j = mcur + tid; j < n; j += kThreads) extra |= kept(j) ? 1 : 0;
+    for (int j = mcur + tid; j < n; j += NT) extra |= kept(j) ? 1 : 0;
     if (__syncthreads_or(extra) && tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_POSITIONS);
     if (tid == 0) p.len[ui.cache_unit] = bud;
     if constexpr (kPaged) {  // pages past the one holding slot bud go back to the pool
@@ -649,7 +699,9 @@ cudaError_t launch_t(const EvictParams &prm, int units, bool fill, cudaStream_t 
     // A programmatic dependent of the previous kernel (the decode step): the kernels wait for it
     // before their first read, and a launch without that attribute is the fallback.
     const bool wide = !fill && units <= BulkRing<T, D>::kCtasPerSm * sm_count();
-    void (*kern)(EvictParams) = fill ? evict_fill_kernel<T, D, kPaged>
+    const bool fill_wide = fill && units <= FillShape<kThreads>::kCtasPerSm * sm_count();
+    void (*kern)(EvictParams) = fill ? (fill_wide ? evict_fill_kernel<T, D, kPaged, kThreads>
+                                                  : evict_fill_kernel<T, D, kPaged, 192>)
                                      : (wide ? evict_kernel<T, D, kPaged, true> : evict_kernel<T, D, kPaged, false>);
     if (wide) {  // above the default 48 KB of dynamic shared memory: opt in once
         static bool configured = false;
@@ -663,7 +715,7 @@ cudaError_t launch_t(const EvictParams &prm, int units, bool fill, cudaStream_t 
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)units, 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.blockDim = dim3(fill && !fill_wide ? 192 : kThreads, 1, 1);
     cfg.dynamicSmemBytes = wide ? BulkRing<T, D>::kBytes : 0;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];

@@ -88,7 +88,7 @@ def gpu_run(w, inp, sample, steps=None, anchors=None, policy=None):
     holds history (bool), compaction ("ordered" / "fill"), budget_bl ([B][L] budgets) and pages
     (a paged cache of that many pages)."""
     S = w.steps if steps is None else steps
-    dev = inp["k_pre"].device
+    dev = inp["q"].device   # the prefill may be in pinned host memory
     B, L, Hq, H, D, G = w.batch, w.layers, w.q_heads, w.kv_heads, w.head_dim, w.group
     pol = policy or {}
     cap = w.capacity if pol.get("pages") is None else (w.capacity + 63) // 64 * 64   # paged: whole pages

@@ -78,6 +78,23 @@ def test_full_size_sampled_units(name, k, steps):
     _pipeline(w, sample_k=k, steps=steps)
 
 
+@pytest.mark.parametrize("name", ["stress", "tiny"])
+def test_stage1_from_pinned_host_prefill(name):
+    """Stage 1 with the prefilled K/V left in pinned host memory: the kernels read the rows over the
+    host link (no device copy of the prompt). The rows, positions and slot maps are the oracle's,
+    bit for bit, and decoding on from that cache matches it too."""
+    w = W.CONFIGS[name] if name == "tiny" else W.scaled(W.CONFIGS[name], layers=2, batch=2, steps=64,
+                                                          name="stress_l2b2")
+    inp = make_inputs(w, "cuda")
+    for key in ("k_pre", "v_pre"):
+        inp[key] = inp[key].cpu().pin_memory()
+    sample = sample_units(w, 10 ** 6)
+    rec = gpu_run(w, inp, sample)
+    check_stage1(w, inp, rec, sample)
+    diverged = check_units(w, rec, oracle_units(w, inp, sample), sample)
+    assert not diverged, diverged
+
+
 # ----------------------------------------------------------------------------- isolated states
 
 def _random_state(desc, lens, seed):
