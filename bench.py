@@ -270,14 +270,20 @@ class Runner:
         s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
         self.graph.replay()
 
-    def request(self, timers=None, lengths=None, evict_timers=None, moved=None, pages=None):
+    def request(self, timers=None, lengths=None, evict_timers=None, moved=None, pages=None, stage1_timers=None):
         """One request: stage 1, then every decode step with evictions. With `timers` (and
         `evict_timers`), records a CUDA event pair around every decode (evict) launch on the launch
         stream. With `moved`, records per eviction the units' lengths and moved rows (this syncs).
         With `pages` (paged cache), records the pages in use after stage 1 and around the first
         eviction (this syncs)."""
         w, s = self.w, self.sess
+        if stage1_timers is not None:
+            s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            s0.record()
         s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
+        if stage1_timers is not None:
+            s1.record()
+            stage1_timers.append((s0, s1))
         if pages is not None:
             from paper_2608_08569_gb300 import paged_pages_in_use
             pages.append(paged_pages_in_use(s.cache))
@@ -602,7 +608,7 @@ def gpu_arm(args, rank, world, local):
         r.request_graph()
     torch.cuda.synchronize()
     barrier(world)
-    timers, ev_timers = [], []
+    timers, ev_timers, st1_timers = [], [], []
     with ClockSampler(local) as clk:
         torch.cuda.synchronize()
         barrier(world)
@@ -613,10 +619,15 @@ def gpu_arm(args, rank, world, local):
             if args.graph and k < args.steps - 1:
                 r.request_graph()
             elif args.graph:  # the last request replays the instrumented copy: per-launch events
+                s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                s0.record()
                 r.sess.prefill(r.k_pre, r.v_pre, *r.span_args[:3], *r.span_args[3:])
+                s1.record()
+                st1_timers.append((s0, s1))
                 r.graph_timed.replay()
             else:
-                r.request(timers=timers, lengths=lengths if k == 0 else None, evict_timers=ev_timers)
+                r.request(timers=timers, lengths=lengths if k == 0 else None, evict_timers=ev_timers,
+                          stage1_timers=st1_timers)
         e1.record()
         torch.cuda.synchronize()
         barrier(world)
@@ -683,6 +694,22 @@ def gpu_arm(args, rank, world, local):
     else:
         roofline_evict = None
 
+    # Stage 1 (span scan, slot map and the fusion kernel, timed together): the prefilled K and V read
+    # once, the stage-1 rows written with their score and position.
+    roofline_stage1 = None
+    if st1_timers and dec_lens:
+        es = 2 if w.dtype == torch.bfloat16 else 4
+        n1 = [x - 1 for x in dec_lens[0]]
+        st1_bytes = w.layers * w.kv_heads * sum(2 * il * w.head_dim * es + nn * (2 * w.head_dim * es + 8)
+                                                for il, nn in zip(w.in_len, n1))
+        st1_ms = sum(a.elapsed_time(b) for a, b in st1_timers) / len(st1_timers)
+        per_req_ms = ms / args.steps
+        roofline_stage1 = {"bound": "hbm", "achieved": round(st1_bytes / (st1_ms / 1000.0) / 1e9, 1), "peak": peak,
+                           "unit": "GB/s", "frac": round(st1_bytes / (st1_ms / 1000.0) / 1e9 / peak, 4),
+                           "kernel": "stage 1: span_scan + slot_map + fuse_rows_kernel (timed together)",
+                           "avg_call_us": round(st1_ms * 1000.0, 1), "alg_bytes_per_call": int(st1_bytes),
+                           "stage1_share_of_step": round(st1_ms / per_req_ms, 4)}
+
     e2e = None
     if not args.no_e2e:
         e2e = e2e_leg(r, args)
@@ -718,7 +745,8 @@ def gpu_arm(args, rank, world, local):
                                             (2 if w.dtype == torch.bfloat16 else 4)},
                    "parallelism": f"replicas x{world} (independent units, no collective)",
                    "l2": "inputs larger than L2 (decode reads ~0.9-7 GB per launch, L2 is 129 MB)"},
-        "roofline": roofline, "roofline_evict": roofline_evict, "gpu_launches": gpu_launches, "clocks": clocks,
+        "roofline": roofline, "roofline_evict": roofline_evict, "roofline_stage1": roofline_stage1,
+        "gpu_launches": gpu_launches, "clocks": clocks,
         "e2e": e2e, "targets": targets,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -631,8 +631,57 @@ __global__ void __launch_bounds__(NT, FillShape<NT>::kCtasPerSm) evict_fill_kern
         return k > thr || (k == thr && (all_ties || q <= pos_thr));
     };
 
-    // Pair the evicted slots below the budget with the kept slots at or above it, in order, a
-    // segment of up to kSegment pairs at a time.
+    // Pair the evicted slots below the budget with the kept slots at or above it, both in ascending
+    // slot order.
+    auto move_pairs = [&](int pairs) {
+        for (int v = tid; v < pairs * 2 * kVecPerRow; v += NT) {
+            const int r = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
+            uint4 *base = w < kVecPerRow ? kc : vc;
+            const int e = w % kVecPerRow;
+            if (VOXZIP_IN_RANGE(p.status, holes[r] >= 0 && holes[r] < bud && movers[r] >= bud && movers[r] < n &&
+                                           row_ok(slot_row(holes[r])) && row_ok(slot_row(movers[r]))))
+                base[slot_row(holes[r]) * kVecPerRow + e] = base[slot_row(movers[r]) * kVecPerRow + e];
+        }
+        for (int r = tid; r < pairs; r += NT) {
+            sc[holes[r]] = sc[movers[r]];
+            ps[holes[r]] = ps[movers[r]];
+        }
+    };
+    // One pass when it fits: each thread classifies a contiguous run of at most 64 slots into a bit
+    // mask, and one block scan per region gives every hole and every mover its rank.
+    {
+        const int ch = (bud + NT - 1) / NT, cm = (n - bud + NT - 1) / NT;
+        int fast = ch <= 64 && cm <= 64;
+        int nh = 0, nm = 0;
+        if (fast) {
+            uint64_t hmask = 0, mmask = 0;
+            const int h0 = tid * ch, m0 = bud + tid * cm;
+            for (int i = 0; i < ch && h0 + i < bud; ++i)
+                if (!kept(h0 + i)) hmask |= 1ull << i;
+            for (int i = 0; i < cm && m0 + i < n; ++i)
+                if (kept(m0 + i)) mmask |= 1ull << i;
+            const int hr = scan_excl<NT>(__popcll(hmask), &nh, warp_sums);
+            const int mr = scan_excl<NT>(__popcll(mmask), &nm, warp_sums);
+            fast = nh <= kSegment && nm <= kSegment;  // the same decision in every thread
+            if (fast) {
+                for (int k = hr; hmask; hmask &= hmask - 1) holes[k++] = h0 + __ffsll((long long)hmask) - 1;
+                for (int k = mr; mmask; mmask &= mmask - 1) movers[k++] = m0 + __ffsll((long long)mmask) - 1;
+            }
+            __syncthreads();
+        }
+        if (fast) {
+            // equal when positions are unique (then exactly `bud` rows are kept)
+            if (nh != nm && tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_POSITIONS);
+            move_pairs(min(nh, nm));
+            __syncthreads();
+            if (tid == 0) p.len[ui.cache_unit] = bud;
+            if constexpr (kPaged) {  // pages past the one holding slot bud go back to the pool
+                if (tid < 32) return_pages_warp(p.pv, ui.cache_unit, bud / kPageTokens + 1, n / kPageTokens + 1);
+            }
+            return;
+        }
+    }
+    // Otherwise a segment of up to kSegment pairs at a time.
     int hcur = 0, mcur = bud;
     while (true) {
         int nh = 0;
@@ -667,18 +716,7 @@ __global__ void __launch_bounds__(NT, FillShape<NT>::kCtasPerSm) evict_fill_kern
         __syncthreads();
         const int pairs = min(nh, nm);  // equal when positions are unique (then exactly `bud` rows are kept)
         if (pairs < nh && tid == 0) raise_status(p.status, VOXZIP_DEV_BAD_POSITIONS);
-        for (int v = tid; v < pairs * 2 * kVecPerRow; v += NT) {
-            const int r = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
-            uint4 *base = w < kVecPerRow ? kc : vc;
-            const int e = w % kVecPerRow;
-            if (VOXZIP_IN_RANGE(p.status, holes[r] >= 0 && holes[r] < bud && movers[r] >= bud && movers[r] < n &&
-                                           row_ok(slot_row(holes[r])) && row_ok(slot_row(movers[r]))))
-                base[slot_row(holes[r]) * kVecPerRow + e] = base[slot_row(movers[r]) * kVecPerRow + e];
-        }
-        for (int r = tid; r < pairs; r += NT) {
-            sc[holes[r]] = sc[movers[r]];
-            ps[holes[r]] = ps[movers[r]];
-        }
+        move_pairs(pairs);
         __syncthreads();
         if (pairs < nh) break;
     }
