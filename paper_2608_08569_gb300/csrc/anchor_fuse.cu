@@ -318,10 +318,21 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
         const int32_t *send = ws.slot_end + (int64_t)b * stride;
         const int32_t *anc = ws.slot_anchor + (int64_t)b * stride;
         const int slot0 = chunk * kSlotsPerPass + warp * kSlotsPerWarp * kRowsPerWarp;
+        // The warp's slots' source ranges and anchor rows, one slot per lane, fetched together up
+        // front, so no slot's row loads wait behind its own metadata load.
+        static_assert(kSlotsPerWarp * kRowsPerWarp <= 32, "one slot per lane");
+        int32_t m0 = 0, m1 = 0, ma = -1;
+        if (lane < kSlotsPerWarp * kRowsPerWarp && slot0 + lane < out_len) {
+            m0 = src[slot0 + lane];
+            m1 = send[slot0 + lane];
+            ma = anc[slot0 + lane];
+        }
         for (int k = 0; k < kSlotsPerWarp; ++k) {
-            const int s = slot0 + k * kRowsPerWarp + sub;
-            if (s >= out_len) break;
-            const int32_t r0 = src[s], r1 = send[s];
+            const int li = k * kRowsPerWarp + sub;
+            const int s = slot0 + li;
+            const int32_t r0 = __shfl_sync(0xffffffffu, m0, li), r1 = __shfl_sync(0xffffffffu, m1, li);
+            const int32_t a_row = __shfl_sync(0xffffffffu, ma, li);
+            if (s >= out_len) continue;  // (every lane still takes the shuffles of every k)
             if (!VOXZIP_IN_RANGE(ws.status, r0 >= 0 && r0 < r1 && r1 <= stride && s < C)) continue;
             float sk[kElems], sv[kElems];
 #pragma unroll
@@ -352,7 +363,6 @@ fuse_rows_kernel(int32_t B, int32_t L, int32_t Hkv, int32_t C, int32_t stride, i
                     sv[i] = __fdiv_rn(sv[i], cnt);
                 }
             }
-            const int32_t a_row = anc[s];
             if (anchor_k != nullptr && a_row >= 0 && VOXZIP_IN_RANGE(ws.status, a_row < anchor_stride)) {
                 float ak[kElems], av[kElems];
 #pragma unroll

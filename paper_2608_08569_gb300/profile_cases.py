@@ -82,6 +82,13 @@ def run(mode: str, reps: int = 6) -> None:
                                i32(sp.off), i32(sp.start), i32(sp.end), i32(sp.groups), c["k"], c["v"], c["score"],
                                c["pos"], c["len"])
             torch.cuda.synchronize()
+        # Algorithmic bytes of the fusion kernel: the prefill K and V read once, the stage-1 rows
+        # written with their score and position.
+        n1 = c["len"][:, 0, 0].long().cpu().tolist()
+        e = 2 if w.dtype == torch.bfloat16 else 4
+        alg = w.layers * w.kv_heads * sum(2 * il * w.head_dim * e + nn * (2 * w.head_dim * e + 8)
+                                          for il, nn in zip(w.in_len, n1))
+        print("algorithmic_bytes_per_launch", int(alg))
     else:
         raise SystemExit(f"unknown case {mode!r}: decode, evict, evict_small or fuse")
     if voxzip_get_status() != 0:
