@@ -3,6 +3,7 @@
     python -m paper_2608_08569_gb300.profile_cases decode [reps]   # decode step, 60-min 20x steady state
     python -m paper_2608_08569_gb300.profile_cases evict [reps]    # one eviction of that state
     python -m paper_2608_08569_gb300.profile_cases evict_small [reps]  # eviction, 10-min 4x steady state
+    python -m paper_2608_08569_gb300.profile_cases evict_fill [reps]   # hole-filling eviction, 60-min 20x
     python -m paper_2608_08569_gb300.profile_cases fuse [reps]     # stage 1 of the 60-min request, 4 layers
 
 Each case holds at most a few GB on the device (decode / evict: 0.94 GB of K/V, 4 sequences x 48
@@ -16,14 +17,14 @@ import numpy as np
 import torch
 
 from . import (CacheDesc, allocate_cache, voxzip_anchor_fuse, voxzip_decode_step, voxzip_evict,
-               voxzip_get_status)
+               voxzip_evict_ex, voxzip_get_status)
 from . import workloads as W
 
 
 def run(mode: str, reps: int = 6) -> None:
     g = torch.Generator(device="cuda")
     g.manual_seed(1)
-    if mode in ("decode", "evict", "evict_small"):
+    if mode in ("decode", "evict", "evict_small", "evict_fill"):
         B, L, Hq, H, D = (1 if mode == "evict_small" else 4), 48, 32, 4, 128
         # 60-min 20x: budget 2 301, up to 32 steps past it; 10-min 4x: budget 2 003
         budget = 2003 if mode == "evict_small" else 2301
@@ -51,6 +52,8 @@ def run(mode: str, reps: int = 6) -> None:
             if mode == "decode":
                 voxzip_decode_step(desc, 0, L, q, kn, vn, npos, c["k"], c["v"], c["score"], c["pos"], c["len"], 0.995,
                                    out, max_len=n + 1)
+            elif mode == "evict_fill":
+                voxzip_evict_ex(desc, 0, L, c["k"], c["v"], c["score"], c["pos"], c["len"], bud, compaction="fill")
             else:
                 voxzip_evict(desc, 0, L, c["k"], c["v"], c["score"], c["pos"], c["len"], bud)
             torch.cuda.synchronize()
@@ -90,7 +93,7 @@ def run(mode: str, reps: int = 6) -> None:
                                           for il, nn in zip(w.in_len, n1))
         print("algorithmic_bytes_per_launch", int(alg))
     else:
-        raise SystemExit(f"unknown case {mode!r}: decode, evict, evict_small or fuse")
+        raise SystemExit(f"unknown case {mode!r}: decode, evict, evict_small, evict_fill or fuse")
     if voxzip_get_status() != 0:
         raise SystemExit("device status word set")
     print("ok", mode)
