@@ -186,3 +186,24 @@ def test_embed_fuse_is_validated(L, d_model, dtype, keep):
 @pytest.mark.parametrize("limit", [0, (1 << 20) + 1])
 def test_selftest_limit_is_validated(L, limit):
     assert L.voxzip_selftest_bounded_wait(limit, None) == 1
+
+
+@pytest.mark.parametrize("ptr,nbytes,sink", [(0, 256, 256), (264, 256, 256), (256, 100, 256), (256, 256, 0)])
+def test_stream_read_is_validated(L, ptr, nbytes, sink):
+    """The streaming-read measurement helper rejects a null or unaligned buffer, a size that is not
+    a multiple of 16 and a null sink before touching the device."""
+    assert L.voxzip_stream_read(ctypes.c_void_p(ptr) if ptr else None, nbytes,
+                                ctypes.c_void_p(sink) if sink else None, None) == 1
+
+
+def test_prefill_may_be_pinned_host_memory_other_tensors_not():
+    """The binding accepts the prefilled K/V in pinned host memory (stage 1 then streams them over
+    the host link) and still demands device tensors for every other argument."""
+    import torch
+    from paper_2608_08569_gb300 import _native as N
+    if not torch.cuda.is_available():
+        # without a CUDA runtime no host memory can be pinned; the check on a plain CPU tensor stands
+        with pytest.raises(ValueError, match="pinned host memory"):
+            N._need(torch.zeros(4, dtype=torch.bfloat16), "k_prefill", torch.bfloat16, pinned_ok=True)
+    with pytest.raises(ValueError, match="on a CUDA device"):
+        N._need(torch.zeros(4, dtype=torch.int32), "in_len", torch.int32)
