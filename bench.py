@@ -483,7 +483,7 @@ def flushed_evict(w, device, peak, flush, fill=False, NL=6):
     return res
 
 
-def decode_loop(w, r, device, NL=32):
+def decode_loop(w, r, device, peak, NL=32):
     """Back-to-back decode launches from one CUDA graph (each a programmatic dependent of the one
     before, no flush: the cache stays in L2 when it fits, as in a serving loop), against the same
     loop of plain streaming reads of the same bytes (voxzip_stream_read): the most a loop of
@@ -512,9 +512,12 @@ def decode_loop(w, r, device, NL=32):
         raise RuntimeError("device status word set by the decode loop")
     t_rd = statistics.median(_graph_replay_ms(rd)[0]) * 1000.0 / NL
     del c, buf
-    return {"us_per_step": round(t_dec, 2), "gbs": round(nbytes / t_dec / 1e3, 1),
+    gbs = nbytes / t_dec / 1e3
+    cache_mb = w.units * (n0 + NL) * 4 * w.head_dim / 1e6   # K and V (bf16) the loop streams
+    return {"us_per_step": round(t_dec, 2), "gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
             "read_us_per_step": round(t_rd, 2), "read_gbs": round(nbytes / t_rd / 1e3, 1),
-            "frac_of_read": round(t_rd / t_dec, 4), "launches": NL, "n_start": n0 + 1}
+            "frac_of_read": round(t_rd / t_dec, 4), "launches": NL, "n_start": n0 + 1,
+            "l2_resident": cache_mb < 64.0}
 
 
 def request_view(r, peak, reps=2):
@@ -572,7 +575,7 @@ def targets_leg(main, device, peak, compaction="ordered", main_request=None):
         res[label] = {
             "workload": name, "budget": max(w.budget),
             "decode": {"request": dec_req, "flushed": flushed_decode(w, r, device, peak, flush),
-                       "loop": decode_loop(w, r, device)},
+                       "loop": decode_loop(w, r, device, peak)},
             "evict": {"request": ev_req, "flushed": flushed_evict(w, device, peak, flush,
                                                                   fill=compaction == "fill")},
         }
@@ -587,8 +590,10 @@ def targets_leg(main, device, peak, compaction="ordered", main_request=None):
                    "evict: budget + interval), a read-only 1 GiB pass before each launch, median of 12-16 "
                    "launches: the HBM-bound number",
         "loop": "32 decode launches back to back from one CUDA graph (programmatic dependent launches, no "
-                "flush), against the same loop of plain streaming reads of the same bytes "
-                "(voxzip_stream_read); frac_of_read = read time / decode time",
+                "flush), as in the request's graph loop but without the per-launch events: frac = algorithmic "
+                "bytes / time against the HBM peak (an effective rate where the cache stays in L2, "
+                "l2_resident), frac_of_read = the same loop of plain streaming reads of the same bytes "
+                "(voxzip_stream_read) / the decode loop",
         "target": f">= {TARGET_FRAC} of the measured HBM peak ({peak} GB/s)"}
     return res
 
