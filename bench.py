@@ -255,14 +255,15 @@ class Runner:
     def capture(self):
         """Captures the decode loop twice after a stage 1: `graph` as it runs (back-to-back launches,
         each a programmatic dependent of the one before), and `graph_timed` with timing events
-        around every launch (events between launches also separate them), for the roofline."""
+        around every eviction and around each run of decode launches between two evictions (the
+        decode launches of a run still overlap one another), for the rooflines."""
         w, s = self.w, self.sess
         s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
         self.graph = s.capture_loop(self.q, self.kn, self.vn, self.npos, self.out, w.interval)
         s.prefill(self.k_pre, self.v_pre, *self.span_args[:3], *self.span_args[3:])
         self.graph_events = []
         self.graph_timed = s.capture_loop(self.q, self.kn, self.vn, self.npos, self.out, w.interval,
-                                          launch_events=self.graph_events)
+                                          launch_events=self.graph_events, segments=True)
 
     def request_graph(self):
         """One request with the decode loop replayed from the graph."""
@@ -322,6 +323,19 @@ class Runner:
                     evict_timers.append((f0, f1))
                 if moved is not None:
                     moved.append(moved_rows(pos_before, n_before, s.cache["pos"], s.cache["len"]))
+
+
+def launch_durations(events):
+    """Per-launch durations (ms) of decode and eviction launches from an instrumented graph's events:
+    a run of decode launches timed as one segment counts its time evenly over its launches."""
+    dec, ev = [], []
+    for kind, a, b, count in events:
+        t = a.elapsed_time(b)
+        if kind == "decode":
+            dec += [t / count] * count
+        else:
+            ev.append(t)
+    return dec, ev
 
 
 def moved_rows(pos_before, n_before, pos_after, n_after):
@@ -534,8 +548,9 @@ def request_view(r, peak, reps=2):
         r.sess.prefill(r.k_pre, r.v_pre, *r.span_args[:3], *r.span_args[3:])
         r.graph_timed.replay()
         torch.cuda.synchronize()
-        dec_t += [a.elapsed_time(b) for kind, a, b in r.graph_events if kind == "decode"]
-        ev_t += [a.elapsed_time(b) for kind, a, b in r.graph_events if kind == "evict"]
+        d, e = launch_durations(r.graph_events)
+        dec_t += d
+        ev_t += e
     dec_lens = [n for kind, n in lengths if kind == "decode"]
     dec_bytes = sum(decode_bytes(w, n) for n in dec_lens) * reps
     ev_bytes = sum(evict_bytes(w, nb, mv) for nb, mv in moved) * reps
@@ -572,6 +587,8 @@ def targets_leg(main, device, peak, compaction="ordered", main_request=None):
         else:
             r.request()   # warm-up
             dec_req, ev_req = request_view(r, peak)
+        # a cache of at most 64 MB stays in L2 from launch to launch: its rate there is effective
+        dec_req["l2_resident"] = w.units * (max(w.budget) + w.interval) * 4 * w.head_dim / 1e6 < 64.0
         res[label] = {
             "workload": name, "budget": max(w.budget),
             "decode": {"request": dec_req, "flushed": flushed_decode(w, r, device, peak, flush),
@@ -583,9 +600,9 @@ def targets_leg(main, device, peak, compaction="ordered", main_request=None):
     del runners
     res["how"] = {
         "request": "the workload's request (stage 1 + every decode step + evictions) replayed from the "
-                   "instrumented CUDA graph, CUDA events around every launch, L2 not flushed (a 10-min "
-                   "cache of 43-203 MB stays partly in L2 between launches); algorithmic bytes from the "
-                   "request's lengths and moved rows",
+                   "instrumented CUDA graph (events around each eviction and around each run of decode launches "
+                   "between two evictions), L2 not flushed (a 10-min cache of 43-203 MB stays partly in L2 "
+                   "between launches); algorithmic bytes from the request's lengths and moved rows",
         "flushed": "one launch at a time at the steady state (decode: budget + interval/2 rows per unit; "
                    "evict: budget + interval), a read-only 1 GiB pass before each launch, median of 12-16 "
                    "launches: the HBM-bound number",
@@ -636,9 +653,12 @@ def gpu_arm(args, rank, world, local):
         e1.record()
         torch.cuda.synchronize()
         barrier(world)
-    if args.graph:  # per-launch times of the instrumented replay, as if every replay took them
-        timers = [(a, b) for kind, a, b in r.graph_events if kind == "decode"] * args.steps
-        ev_timers = [(a, b) for kind, a, b in r.graph_events if kind == "evict"] * args.steps
+    if args.graph:  # launch times of the instrumented replay, as if every replay took them
+        dec_dur, ev_dur = launch_durations(r.graph_events)
+        dec_dur, ev_dur = dec_dur * args.steps, ev_dur * args.steps
+    else:
+        dec_dur = [a.elapsed_time(b) for a, b in timers]
+        ev_dur = [a.elapsed_time(b) for a, b in ev_timers]
     ms = e0.elapsed_time(e1)
     ms_max = max_over_ranks(ms, world)
     total_steps = world * args.steps * w.steps
@@ -647,8 +667,8 @@ def gpu_arm(args, rank, world, local):
     # Roofline of the dominant kernel (the decode step): algorithmic bytes over event-timed duration.
     dec_lens = [n for kind, n in lengths if kind == "decode"]
     bytes_per_request = sum(decode_bytes(w, n) for n in dec_lens)
-    dec_ms = sum(a.elapsed_time(b) for a, b in timers)
-    launches = len(timers)
+    dec_ms = sum(dec_dur)
+    launches = len(dec_dur)
     avg_ms = dec_ms / launches
     achieved = bytes_per_request * args.steps / (dec_ms / 1000.0) / 1e9
     peak, peak_kind = peaks()
@@ -666,11 +686,11 @@ def gpu_arm(args, rank, world, local):
                 "alg_bytes_per_launch": int(bytes_per_request / max(1, len(dec_lens))),
                 "decode_share_of_step": round(dec_ms / ms, 4)}
     # The same split at the first eviction: before it the cache holds the whole stage-1 output.
-    pre = [i for i in range(len(timers)) if i % w.steps < w.interval]
-    post = [i for i in range(len(timers)) if i % w.steps >= w.interval]
+    pre = [i for i in range(len(dec_dur)) if i % w.steps < w.interval]
+    post = [i for i in range(len(dec_dur)) if i % w.steps >= w.interval]
     for name, ids in (("before_first_evict", pre), ("after_first_evict", post)):
         b = sum(decode_bytes(w, dec_lens[i % w.steps]) for i in ids)
-        t = sum(timers[i][0].elapsed_time(timers[i][1]) for i in ids)
+        t = sum(dec_dur[i] for i in ids)
         if t > 0:
             roofline[f"achieved_{name}"] = round(b / (t / 1000.0) / 1e9, 1)
     # kernels per request: 3 stage-1 kernels (5 paged), one decode launch per step, one evict per interval
@@ -681,8 +701,8 @@ def gpu_arm(args, rank, world, local):
     r.request(moved=moved, pages=pages)
     torch.cuda.synchronize()
     ev_bytes = sum(evict_bytes(w, nb, mv) for nb, mv in moved)
-    ev_ms = sum(a.elapsed_time(b) for a, b in ev_timers)
-    if ev_timers and ev_ms > 0:
+    ev_ms = sum(ev_dur)
+    if ev_dur and ev_ms > 0:
         ev_ach = ev_bytes * args.steps / (ev_ms / 1000.0) / 1e9
         etr = profiled_traffic_ratio("evict_kernel_stress.md", ["evict.cu", "common.cuh"]) \
             if args.compaction == "ordered" else None
@@ -693,7 +713,7 @@ def gpu_arm(args, rank, world, local):
                           "kernel": "evict_kernel (top-N select + ordered in-place compaction)"
                           if args.compaction == "ordered" else
                           "evict_fill_kernel (top-N select + hole-filling compaction)",
-                          "avg_launch_us": round(1000.0 * ev_ms / len(ev_timers), 2),
+                          "avg_launch_us": round(1000.0 * ev_ms / len(ev_dur), 2),
                           "alg_bytes_per_launch": int(ev_bytes / max(1, len(moved))),
                           "evict_share_of_step": round(ev_ms / ms, 4)}
     else:
@@ -736,9 +756,11 @@ def gpu_arm(args, rank, world, local):
                    "gamma": w.gamma, "decode_steps_per_request": w.steps, "evict_interval": w.interval,
                    "compaction": args.compaction, "graph": bool(args.graph),
                    "loop": "graph" if args.graph else "eager",
-                   "roofline_timing": ("CUDA events around every launch of the last timed request, which "
-                                       "replays an instrumented copy of the graph (events between launches "
-                                       "keep them from overlapping, so the others replay without)")
+                   "roofline_timing": ("CUDA events in the last timed request, which replays an instrumented "
+                                       "copy of the graph: around every eviction, and around each run of 32 "
+                                       "decode launches between two evictions (the decode launches of a run "
+                                       "overlap one another as in the plain graph); a run's time counts evenly "
+                                       "over its launches")
                                       if args.graph else
                                       "CUDA events around every launch inside the timed region",
                    "paged": None if not args.paged else {

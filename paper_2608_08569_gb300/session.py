@@ -94,40 +94,47 @@ class Session:
             self.n_max = min(self.n_max, max(self.budget_host))
 
     # decode loop in a CUDA graph ---------------------------------------------------------------------
-    def capture_loop(self, q, k_new, v_new, new_pos, out, interval: int, *, launch_events=None):
+    def capture_loop(self, q, k_new, v_new, new_pos, out, interval: int, *, launch_events=None,
+                     segments: bool = False):
         """Captures the decode loop of one request: step t (1-based) decodes with q[t-1], k_new[t-1],
         v_new[t-1], new_pos[t-1] into out[t-1], and evicts when t % interval == 0. Call it right
         after a prefill of the request's shape (it starts from that cache length bound); replaying
         the returned graph after each later prefill of the same shape runs the whole loop with one
-        host call. With `launch_events` (a list), a pair of timing events (created with
-        external=True) around every decode and every eviction launch is captured too and appended
-        as ("decode" | "evict", start, end); the graph records into them on every replay, so they
-        must outlive it."""
+        host call. With `launch_events` (a list), timing events (created with external=True) are
+        captured too and appended as (kind, start, end, launches): around every decode launch
+        ("decode", ..., 1), or with `segments` around each run of decode launches between two
+        evictions ("decode", ..., steps in the run: the launches keep overlapping one another as in
+        the plain graph), and around every eviction ("evict", ..., 1). The graph records into them
+        on every replay, so they must outlive it."""
         n0 = self.n_max
         stream = torch.cuda.Stream(device=self.device)
         stream.wait_stream(torch.cuda.current_stream(self.device))
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.stream(stream):
             with torch.cuda.graph(graph, stream=stream):
-                for t in range(1, q.shape[0] + 1):
-                    ev = None
-                    if launch_events is not None:
-                        ev = (torch.cuda.Event(enable_timing=True, external=True),
+                steps = q.shape[0]
+                mk = lambda: (torch.cuda.Event(enable_timing=True, external=True),
                               torch.cuda.Event(enable_timing=True, external=True))
+                ev, run = None, 0
+                for t in range(1, steps + 1):
+                    if launch_events is not None and ev is None:
+                        ev = mk()
                         ev[0].record()
                     self.decode(q[t - 1], k_new[t - 1], v_new[t - 1], new_pos[t - 1], out[t - 1])
-                    if ev is not None:
+                    run += 1
+                    if ev is not None and (not segments or t % interval == 0 or t == steps):
                         ev[1].record()
-                        launch_events.append(("decode",) + ev)
+                        launch_events.append(("decode", ev[0], ev[1], run))
+                        ev, run = None, 0
                     if t % interval == 0:
+                        eev = None
                         if launch_events is not None:
-                            ev = (torch.cuda.Event(enable_timing=True, external=True),
-                                  torch.cuda.Event(enable_timing=True, external=True))
-                            ev[0].record()
+                            eev = mk()
+                            eev[0].record()
                         self.evict()
-                        if launch_events is not None:
-                            ev[1].record()
-                            launch_events.append(("evict",) + ev)
+                        if eev is not None:
+                            eev[1].record()
+                            launch_events.append(("evict", eev[0], eev[1], 1))
         torch.cuda.current_stream(self.device).wait_stream(stream)
         self.n_max = n0
         return graph
