@@ -536,7 +536,8 @@ def decode_loop(w, r, device, peak, NL=32):
 
 def request_view(r, peak, reps=2):
     """The decode and evict kernels as they run in the workload's request (stage 1, then the decode
-    loop replayed from the instrumented CUDA graph, events around every launch, no flush)."""
+    loop replayed from the instrumented CUDA graph: events around every eviction and every run of
+    decode launches between two evictions, no flush)."""
     w = r.w
     lengths, moved = [], []
     r.request(lengths=lengths)
@@ -640,7 +641,7 @@ def gpu_arm(args, rank, world, local):
         for k in range(args.steps):
             if args.graph and k < args.steps - 1:
                 r.request_graph()
-            elif args.graph:  # the last request replays the instrumented copy: per-launch events
+            elif args.graph:  # the last request replays the instrumented copy (events per run of launches)
                 s0, s1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 s0.record()
                 r.sess.prefill(r.k_pre, r.v_pre, *r.span_args[:3], *r.span_args[3:])
