@@ -17,6 +17,11 @@ captured once, each launch a programmatic dependent of the one before; stage 1 r
 audio to spans (Eq. 3, on the host) and the fusion of the prompt embeddings (d_model 2048) with the
 embedded transcriptions as anchors; one step fuses the four sequences once.
 
+The JSON line also carries the decode, eviction and stage-1 rooflines, the decode and eviction
+kernels at the four target points (60-min and 10-min audio, each at the 20x and 4x budgets:
+`targets`), the end-to-end rate from pinned host memory (`e2e`) and the oracle's rate on the host
+cores (`cpu_baseline`).
+
 Under torchrun each rank runs its own replica of the workload on its own GPU (the units of the
 path are independent, so there is no data-path collective); the time is the max over ranks.
 `--impl reference` times the fp64 CPU oracle on a bounded sample of the same workload instead.

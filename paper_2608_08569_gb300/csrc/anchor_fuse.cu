@@ -13,7 +13,9 @@
 //               kv-head) unit (a lane owns one 16-byte vector of the row; four source rows in
 //               flight): the fp32 mean of the slot's source rows (a copy when the range has one
 //               row) plus the anchor row, rounded once to the cache dtype; K and V in the same
-//               pass; pos and score = 0;
+//               pass; pos and score = 0. A persistent grid walks (128-slot chunk, unit) items;
+//               prefill rows in pinned host memory are streamed over the host link by CTAs on
+//               half the SMs;
 //   fuse_wide   embedding level, any width that is a whole number of 16-byte vectors: one warp per
 //               output row of a sequence, the same arithmetic.
 // Output slots cover the kept tokens of the prompt in order, each a contiguous source range.

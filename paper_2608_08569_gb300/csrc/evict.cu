@@ -28,11 +28,13 @@
 //              and each sub-chunk's moving rows out, by 1-D bulk copies.
 //
 // evict_fill_kernel (hole filling): sinks are the T lowest positions and the recent window the M
-// highest (radix selects over the positions), so the cache need not be in time order; the
+// highest (both cuts in one radix sweep per digit), so the cache need not be in time order; the
 // history select is the same. Kept rows below the budget stay; the kept rows at slots >= budget
 // move, in ascending slot order, into the evicted slots below the budget, in ascending slot
 // order: at most n - budget rows move. Sources lie at or above the budget and destinations below
-// it, so no copy can read a row another one wrote.
+// it, so no copy can read a row another one wrote. Its time is the latency of its passes, so the
+// block size follows the unit count: 256 threads when the launch fits one wave of 4 CTAs per SM,
+// else 192 threads (6 per SM).
 #include "common.cuh"
 #include "evict_policy.cuh"
 #include "paged.cuh"
