@@ -634,15 +634,29 @@ __global__ void __launch_bounds__(NT, FillShape<NT>::kCtasPerSm) evict_fill_kern
     };
 
     // Pair the evicted slots below the budget with the kept slots at or above it, both in ascending
-    // slot order.
+    // slot order. Sources lie at or above the budget and destinations below it, so a thread loads all
+    // of its vectors of a round (kBatch of them) before it stores any.
     auto move_pairs = [&](int pairs) {
-        for (int v = tid; v < pairs * 2 * kVecPerRow; v += NT) {
-            const int r = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
-            uint4 *base = w < kVecPerRow ? kc : vc;
-            const int e = w % kVecPerRow;
-            if (VOXZIP_IN_RANGE(p.status, holes[r] >= 0 && holes[r] < bud && movers[r] >= bud && movers[r] < n &&
-                                           row_ok(slot_row(holes[r])) && row_ok(slot_row(movers[r]))))
-                base[slot_row(holes[r]) * kVecPerRow + e] = base[slot_row(movers[r]) * kVecPerRow + e];
+        constexpr int kBatch = 4;
+        const int total = pairs * 2 * kVecPerRow;
+        for (int v0 = tid; v0 < total; v0 += kBatch * NT) {
+            uint4 x[kBatch];
+            bool go[kBatch];
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u) {
+                const int v = v0 + u * NT;
+                const int r = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
+                go[u] = v < total && VOXZIP_IN_RANGE(p.status, holes[r] >= 0 && holes[r] < bud && movers[r] >= bud &&
+                                                                   movers[r] < n && row_ok(slot_row(holes[r])) &&
+                                                                   row_ok(slot_row(movers[r])));
+                if (go[u]) x[u] = (w < kVecPerRow ? kc : vc)[slot_row(movers[r]) * kVecPerRow + w % kVecPerRow];
+            }
+#pragma unroll
+            for (int u = 0; u < kBatch; ++u) {
+                const int v = v0 + u * NT;
+                const int r = v / (2 * kVecPerRow), w = v % (2 * kVecPerRow);
+                if (go[u]) (w < kVecPerRow ? kc : vc)[slot_row(holes[r]) * kVecPerRow + w % kVecPerRow] = x[u];
+            }
         }
         for (int r = tid; r < pairs; r += NT) {
             sc[holes[r]] = sc[movers[r]];
