@@ -219,25 +219,33 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
     const int ntiles = (cnt + kTile - 1) / kTile;
 
     // Eq. 1: the appended row is local row jn of the CTA whose range holds slot n-1. The consumer
-    // warp that owns that row of its tile keeps k_new / v_new in registers, stores them to the cache
-    // for later steps and writes them over the row the TMA brought in, so no load waits for the store.
+    // warp that owns that row of its tile loads k_new / v_new into registers here, writes them over
+    // the row the TMA brought in, so no load waits for the store, and stores them (with the position)
+    // to the cache for later steps when it patches that tile: a store issued here would wait for its
+    // load and hold back the barrier before the ring's first load.
     const int jn = n - 1 - j0;
     const bool own_new = jn >= 0 && jn < cnt;
     const int t_new = own_new ? jn / kTile : -1;
     const bool patcher = own_new && warp == (jn % kTile) / 16;
     const uint32_t patch_off = own_new ? (uint32_t)(lane >> 3) * kBoxBytes + swz(jn % kTile, lane & 7) : 0u;
+    const int64_t drow = kPaged ? (int64_t)page_new * kPageTokens + (n_old & (kPageTokens - 1)) : row_base + n - 1;
     uint4 kn4 = make_uint4(0u, 0u, 0u, 0u), vn4 = make_uint4(0u, 0u, 0u, 0u);
+    int32_t pos_new = 0;
     if (patcher && lane < D / 8) {
         const int64_t src = (act_row * p.Hkv + ui.h) * D + lane * 8;
         kn4 = *reinterpret_cast<const uint4 *>(p.k_new + src);
         vn4 = *reinterpret_cast<const uint4 *>(p.v_new + src);
-        const int64_t drow = kPaged ? (int64_t)page_new * kPageTokens + (n_old & (kPageTokens - 1)) : row_base + n - 1;
-        if (VOXZIP_IN_RANGE(p.status, drow >= 0 && drow < p.rows)) {
+        if (lane == 0) pos_new = p.new_pos[ui.b];
+    }
+    bool appended = false;  // the patcher warp has stored the appended row
+    auto append = [&]() {
+        if (lane < D / 8 && VOXZIP_IN_RANGE(p.status, drow >= 0 && drow < p.rows)) {
             *reinterpret_cast<uint4 *>(p.k_cache + drow * D + lane * 8) = kn4;
             *reinterpret_cast<uint4 *>(p.v_cache + drow * D + lane * 8) = vn4;
         }
-        if (lane == 0) p.pos[row_base + n - 1] = p.new_pos[ui.b];
-    }
+        if (lane == 0) p.pos[row_base + n - 1] = pos_new;
+        appended = true;
+    };
     if (tid == 0) {
         for (int s = 0; s < kStages; ++s) {
             ptx::mbar_init(&full[s], 1);
@@ -322,6 +330,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                 const bool patch = patcher && t == t_new;
                 if (patch) {
                     if (lane < D / 8) *reinterpret_cast<uint4 *>(stage + patch_off) = kn4;
+                    append();
                     __syncwarp();
                 }
                 const uint32_t base = ptx::smem_u32(stage);
@@ -366,6 +375,7 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
             __syncwarp();
             if (lane == 0) ptx::mbar_arrive(&empty[s]);
         }
+        if (patcher && !appended) append();  // phase K ended early (a wait gave up)
         // Per-head statistics of the warp (merge over the 8 lanes that share qd), then of the CTA.
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
@@ -604,9 +614,11 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
             case 8: combine(std::integral_constant<int, 8>{}); break;
             default: combine(std::integral_constant<int, 16>{}); break;
         }
-        // This CTA is done reading its peers' shared memory; they may leave once all have said so.
-        // The score update below touches only this CTA's own shared memory and global memory.
-        asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+        // This CTA is done reading its peers' shared memory (every value read has been used above);
+        // they may leave once all have said so. The arrive orders nothing else, so it is relaxed and
+        // does not wait for the output stores. The score update below touches only this CTA's own
+        // shared memory and global memory.
+        asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
         // Eq. 6 for this CTA's tokens: A = gamma * [A, 0] + sum over the group's heads.
         const float *fs = fac + rank * GP;
         float *sc = p.score + row_base + j0;
