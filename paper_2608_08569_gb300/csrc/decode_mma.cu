@@ -334,9 +334,13 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                     __syncwarp();
                 }
                 const uint32_t base = ptx::smem_u32(stage);
-                float acc[NT][4];
+                // Two accumulators (even and odd k-steps), summed at the end: two independent mma
+                // chains of half the length on the per-tile critical path.
+                float acc2[2][NT][4];
 #pragma unroll
-                for (int nt = 0; nt < NT; ++nt) acc[nt][0] = acc[nt][1] = acc[nt][2] = acc[nt][3] = 0.f;
+                for (int c = 0; c < 2; ++c)
+#pragma unroll
+                    for (int nt = 0; nt < NT; ++nt) acc2[c][nt][0] = acc2[c][nt][1] = acc2[c][nt][2] = acc2[c][nt][3] = 0.f;
                 const int arow = r0 + (lane & 7) + ((lane >> 3) & 1) * 8;
 #pragma unroll
                 for (int h = 0; h < kHalves; ++h) {
@@ -346,9 +350,15 @@ decode_mma_kernel(const __grid_constant__ CUtensorMap tmk, const __grid_constant
                         ptx::ldsm_x4(base + h * kBoxBytes + swz(arow, kk * 2 + (lane >> 4)), a0, a1, a2, a3);
 #pragma unroll
                         for (int nt = 0; nt < NT; ++nt)
-                            ptx::mma_bf16_16816(acc[nt], a0, a1, a2, a3, qb[nt][h * 4 + kk][0], qb[nt][h * 4 + kk][1]);
+                            ptx::mma_bf16_16816(acc2[kk & 1][nt], a0, a1, a2, a3, qb[nt][h * 4 + kk][0],
+                                                qb[nt][h * 4 + kk][1]);
                     }
                 }
+                float acc[NT][4];
+#pragma unroll
+                for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) acc[nt][e] = acc2[0][nt][e] + acc2[1][nt][e];
                 // acc[nt][2 * half + j]: token lt0 + g + 8 * half, head nt * 8 + 2 * qd + j.
                 const bool va = lt0 + g < cnt, vb = lt0 + g + 8 < cnt;
 #pragma unroll
