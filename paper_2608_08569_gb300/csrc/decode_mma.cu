@@ -19,7 +19,8 @@
 // maximum and normaliser: every CTA rewrites its tokens' scores and combines one slice of the
 // G x D outputs from all CTAs' partials. (Exchanging the statistics between the two phases instead
 // makes every CTA wait twice for the slowest one of its cluster, which measured slower.)
-// The appended row is patched into its tile in shared memory, so no load waits for its store.
+// The appended row is patched into its tile in shared memory, so no load waits for its store; its
+// cache stores go out at that patch, not in the prologue, where they would wait for their loads.
 // Paged caches (kPaged): a CTA's range is whole 64-token pages, each tile is loaded from the pool
 // row its page-table entry gives, and the CTA that completes a page takes the next one.
 #include <cooperative_groups.h>
